@@ -1,0 +1,323 @@
+"""Checks that pin the fp64 oracle to facts outside itself.
+
+Each ``check_*`` function takes the oracle functions it exercises as
+arguments and returns a list of failure messages (empty = pinned).  The pin
+tests call them with the real oracle; the planted-mistake tests call them
+with deliberately broken copies and require a failure, so a plausible slip
+anywhere in the oracle (a dropped scale, a wrong sign, a transposed operand,
+an off-by-one tile, a reversed tie-break) is shown to be caught.
+
+Independent sources used: hand-worked fixtures under tests/golden/, torch's
+CPU scaled_dot_product_attention and autograd in float64, brute-force Python
+loops, closed forms and central finite differences.
+"""
+from __future__ import annotations
+
+import json
+import math
+import os
+
+import numpy as np
+import torch
+import torch.nn.functional as F
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _load(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def _close(a, b, tol=1e-10):
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    return a.shape == b.shape and bool(np.all(np.abs(a - b) <= tol * (1.0 + np.abs(b))))
+
+
+# ------------------------------------------------------------ small inputs
+def random_case(seed=0, N=13, H=2, d=8, b=4, density=0.5, force_nonempty=True):
+    g = np.random.Generator(np.random.PCG64([1234, seed]))
+    q = g.standard_normal((N, H, d))
+    k = g.standard_normal((N, H, d))
+    v = g.standard_normal((N, H, d))
+    do = g.standard_normal((N, H, d))
+    nq = -(-N // b)
+    bm = (g.random((H, nq, nq)) < density).astype(np.uint8)
+    if force_nonempty:
+        for h in range(H):
+            for i in range(nq):
+                if not bm[h, i].any():
+                    bm[h, i, g.integers(nq)] = 1
+    return q, k, v, do, bm
+
+
+def token_mask(bm: np.ndarray, N: int, b: int) -> np.ndarray:
+    """[H, N, N] bool: query token r may see key token c (brute-force expansion)."""
+    H = bm.shape[0]
+    m = np.zeros((H, N, N), dtype=bool)
+    for h in range(H):
+        for r in range(N):
+            for c in range(N):
+                m[h, r, c] = bool(bm[h, r // b, c // b])
+    return m
+
+
+def sdpa_reference(q, k, v, tok_mask, scale, need_grad=False, do=None):
+    """torch SDPA in float64 on CPU; heads as the batch dim."""
+    Q = torch.tensor(q.transpose(1, 0, 2), dtype=torch.float64, requires_grad=need_grad)
+    K = torch.tensor(k.transpose(1, 0, 2), dtype=torch.float64, requires_grad=need_grad)
+    V = torch.tensor(v.transpose(1, 0, 2), dtype=torch.float64, requires_grad=need_grad)
+    M = None if tok_mask is None else torch.tensor(tok_mask)
+    O = F.scaled_dot_product_attention(Q, K, V, attn_mask=M, scale=scale)
+    if not need_grad:
+        return O.detach().numpy().transpose(1, 0, 2)
+    O.backward(torch.tensor(do.transpose(1, 0, 2)))
+    return (O.detach().numpy().transpose(1, 0, 2),
+            Q.grad.numpy().transpose(1, 0, 2), K.grad.numpy().transpose(1, 0, 2),
+            V.grad.numpy().transpose(1, 0, 2))
+
+
+# ---------------------------------------------------------------- compaction
+def check_compaction(fg_compact, fg_scatter, BG_KEEP=0, BG_ZERO=1, BG_FILL=2):
+    bad = []
+    gd = _load("compaction_hand.json")
+    mask = np.array(gd["mask"], np.uint8)
+    rows = np.array(gd["rows"], np.float64)
+    idx, (xc,) = fg_compact(mask, [rows])
+    if list(idx) != gd["idx"]:
+        bad.append(f"hand idx {list(idx)} != {gd['idx']}")
+    if not _close(xc, gd["compacted"]):
+        bad.append("hand compacted rows")
+    src = np.array(gd["scatter_src"], np.float64)
+    for mode, key in ((BG_KEEP, "scatter_keep"), (BG_ZERO, "scatter_zero"), (BG_FILL, "scatter_fill")):
+        y = fg_scatter(np.array(gd["idx"], np.int32), src, rows, mode, np.array(gd["fill_row"], np.float64))
+        if not _close(y, gd[key]):
+            bad.append(f"hand {key}")
+    g = np.random.Generator(np.random.PCG64(7))
+    T = 257
+    x = g.standard_normal((T, 3, 4))
+    # all-foreground: identity
+    idx, (xc,) = fg_compact(np.ones(T, np.uint8), [x])
+    if not (np.array_equal(idx, np.arange(T)) and np.array_equal(xc, x)):
+        bad.append("all-foreground is not the identity")
+    # all-background: empty
+    idx, (xc,) = fg_compact(np.zeros(T, np.uint8), [x])
+    if len(idx) != 0 or xc.shape[0] != 0:
+        bad.append("all-background is not empty")
+    # random: N = popcount, strictly increasing, rows gathered, scatter o gather
+    m = (g.random(T) < 0.37).astype(np.uint8)
+    idx, (xc,) = fg_compact(m, [x])
+    if len(idx) != int(m.sum()):
+        bad.append("N != popcount")
+    if len(idx) > 1 and not np.all(np.diff(idx) > 0):
+        bad.append("idx not strictly increasing")
+    if not all(m[t] for t in idx):
+        bad.append("idx holds a background position")
+    if not all(np.array_equal(xc[n], x[idx[n]]) for n in range(len(idx))):
+        bad.append("compacted row is not the canvas row")
+    y0 = g.standard_normal(x.shape)
+    y = fg_scatter(idx, xc, y0, BG_KEEP)
+    if not (np.array_equal(y[m == 1], x[m == 1]) and np.array_equal(y[m == 0], y0[m == 0])):
+        bad.append("scatter o gather is not identity on fg / untouched on bg")
+    return bad
+
+
+# -------------------------------------------------------------- block lists
+def check_block_lists(bitmap_to_csr, csr_to_csc):
+    bad = []
+    g = np.random.Generator(np.random.PCG64(11))
+    H, nq, nk = 3, 7, 7
+    bm = (g.random((H, nq, nk)) < 0.4).astype(np.uint8)
+    bm[1, 2, :] = 0                                   # an empty row
+    row_ptr, col_idx = bitmap_to_csr(bm)
+    # brute force: Python loops
+    rp, ci = [0], []
+    for h in range(H):
+        for i in range(nq):
+            for j in range(nk):
+                if bm[h, i, j]:
+                    ci.append(j)
+            rp.append(len(ci))
+    if list(row_ptr) != rp or list(col_idx) != ci:
+        bad.append("CSR differs from brute force")
+    col_ptr, row_idx = csr_to_csc(row_ptr, col_idx, H, nq, nk)
+    cp, ri = [0], []
+    for h in range(H):
+        for j in range(nk):
+            for i in range(nq):
+                if bm[h, i, j]:
+                    ri.append(i)
+            cp.append(len(ri))
+    if list(col_ptr) != cp or list(row_idx) != ri:
+        bad.append("CSC differs from brute-force transpose")
+    return bad
+
+
+# ------------------------------------------------------------------- Top-K
+def check_topk(topk_block_mask, block_pool, k_rho):
+    bad = []
+    gd = _load("topk_hand.json")
+    q = np.array(gd["q"], np.float64)[:, None, :]
+    k = np.array(gd["k"], np.float64)[:, None, :]
+    b = gd["block"]
+    pq = block_pool(q[:, 0], b)
+    pk = block_pool(k[:, 0], b)
+    if not _close(pq @ pk.T, gd["scores"]):
+        bad.append("hand S_c")
+    for rho, want in gd["expected"].items():
+        rp, ci, _, kr = topk_block_mask(q, k, b, float(rho))
+        got = [list(ci[rp[r]:rp[r + 1]]) for r in range(len(rp) - 1)]
+        if got != want:
+            bad.append(f"hand Top-K rho={rho}: {got} != {want}")
+    # brute force on random inputs (Python sort on (-score, j))
+    g = np.random.Generator(np.random.PCG64(5))
+    N, H, d, b = 45, 2, 6, 4
+    q = g.standard_normal((N, H, d))
+    k = g.standard_normal((N, H, d))
+    nk = -(-N // b)
+    for rho in (0.05, 0.2, 0.5, 1.0):
+        rp, ci, _, kr = topk_block_mask(q, k, b, rho)
+        if kr != max(1, math.floor(rho * nk)):
+            bad.append(f"K_rho for rho={rho}")
+        for h in range(H):
+            means_q = [q[i * b:min(N, i * b + b), h].sum(0) / len(range(i * b, min(N, i * b + b))) for i in range(nk)]
+            means_k = [k[j * b:min(N, j * b + b), h].sum(0) / len(range(j * b, min(N, j * b + b))) for j in range(nk)]
+            for i in range(nk):
+                s = [float(np.dot(means_q[i], means_k[j])) for j in range(nk)]
+                want = sorted(sorted(range(nk), key=lambda j: (-s[j], j))[:kr])
+                r = h * nk + i
+                if list(ci[rp[r]:rp[r + 1]]) != want:
+                    bad.append(f"brute-force Top-K rho={rho} h={h} i={i}")
+                    break
+    # rho = 1 keeps every block; constant scores keep the first K_rho blocks
+    rp, ci, _, kr = topk_block_mask(q, k, b, 1.0)
+    if kr != nk or not all(list(ci[rp[r]:rp[r + 1]]) == list(range(nk)) for r in range(len(rp) - 1)):
+        bad.append("rho = 1 does not keep every block")
+    z = np.zeros((N, H, d))
+    rp, ci, _, kr = topk_block_mask(z, k, b, 0.3)
+    if not all(list(ci[rp[r]:rp[r + 1]]) == list(range(kr)) for r in range(len(rp) - 1)):
+        bad.append("all-tied scores do not keep the smallest indices")
+    return bad
+
+
+# ---------------------------------------------------------- attention forward
+def check_forward(bsattn_fwd, bitmap_to_csr):
+    bad = []
+    gd = _load("attention_hand.json")
+    q = np.array(gd["q"], np.float64).reshape(-1, 1, 1)
+    k = np.array(gd["k"], np.float64).reshape(-1, 1, 1)
+    v = np.array(gd["v"], np.float64).reshape(-1, 1, 1)
+    b = gd["block"]
+    row_ptr = np.array([0] + list(np.cumsum([len(x) for x in gd["lists"]])), np.int32)
+    col_idx = np.array(sum(gd["lists"], []), np.int32)
+    O, LSE = bsattn_fwd(q, k, v, row_ptr, col_idx, b, gd["scale"])
+    if not _close(O[:, 0, 0], gd["o"]):
+        bad.append(f"hand O {O[:, 0, 0]} != {gd['o']}")
+    if not _close(LSE[0], gd["lse"]):
+        bad.append(f"hand LSE {LSE[0]} != {gd['lse']}")
+
+    for seed, (N, H, d, b, dens) in enumerate([(13, 2, 8, 4, 0.5), (32, 1, 16, 8, 0.3), (9, 3, 4, 3, 0.7)]):
+        q, k, v, _, bm = random_case(seed, N, H, d, b, dens)
+        scale = 1.0 / math.sqrt(d)
+        rp, ci = bitmap_to_csr(bm)
+        O, LSE = bsattn_fwd(q, k, v, rp, ci, b)
+        tm = token_mask(bm, N, b)
+        ref = sdpa_reference(q, k, v, tm, scale)
+        if not _close(O, ref, 1e-10):
+            bad.append(f"masked SDPA mismatch (case {seed})")
+        # rows sum to one: sum_k exp(s - LSE) over the visible keys
+        for h in range(H):
+            s = (q[:, h] @ k[:, h].T) * scale
+            tot = np.where(tm[h], np.exp(s - LSE[h][:, None]), 0.0).sum(1)
+            if not _close(tot, np.ones(N), 1e-12):
+                bad.append(f"softmax rows do not sum to 1 (case {seed})")
+                break
+        # all-ones mask equals dense attention
+        ones = np.ones_like(bm)
+        rp1, ci1 = bitmap_to_csr(ones)
+        O1, _ = bsattn_fwd(q, k, v, rp1, ci1, b)
+        if not _close(O1, sdpa_reference(q, k, v, None, scale), 1e-10):
+            bad.append(f"all-ones mask != dense SDPA (case {seed})")
+        # constant V rows -> O equals the constant
+        cv = np.broadcast_to(np.arange(d, dtype=np.float64), (N, H, d)).copy()
+        Oc, _ = bsattn_fwd(q, k, cv, rp, ci, b)
+        if not _close(Oc, cv, 1e-12):
+            bad.append(f"constant V closed form (case {seed})")
+        # identical K rows (or Q = 0) -> mean of the selected V rows
+        kk = np.broadcast_to(k[:1], k.shape).copy()
+        for qq, kk_, name in ((q, kk, "identical K"), (np.zeros_like(q), k, "Q = 0")):
+            Om, _ = bsattn_fwd(qq, kk_, v, rp, ci, b)
+            want = np.zeros_like(Om)
+            for h in range(H):
+                for r in range(N):
+                    want[r, h] = v[tm[h, r], h].mean(0)
+            if not _close(Om, want, 1e-12):
+                bad.append(f"{name} closed form (case {seed})")
+    # an empty list: O = 0, LSE = -inf, no NaN
+    q, k, v, _, bm = random_case(3, 8, 1, 4, 4, 0.5)
+    bm[0, 1, :] = 0
+    rp, ci = bitmap_to_csr(bm)
+    O, LSE = bsattn_fwd(q, k, v, rp, ci, 4)
+    if not (np.all(O[4:8] == 0) and np.all(np.isneginf(LSE[0, 4:8])) and not np.isnan(O).any()):
+        bad.append("empty key list is not O = 0, LSE = -inf")
+    return bad
+
+
+# --------------------------------------------------------- attention backward
+def check_backward(bsattn_fwd, bsattn_bwd, bitmap_to_csr):
+    bad = []
+    for seed, (N, H, d, b, dens) in enumerate([(13, 2, 8, 4, 0.5), (10, 1, 4, 5, 0.6)]):
+        q, k, v, do, bm = random_case(10 + seed, N, H, d, b, dens)
+        scale = 1.0 / math.sqrt(d)
+        rp, ci = bitmap_to_csr(bm)
+        dQ, dK, dV = bsattn_bwd(q, k, v, do, rp, ci, b)
+        _, gq, gk, gv = sdpa_reference(q, k, v, token_mask(bm, N, b), scale, True, do)
+        for name, a, r in (("dQ", dQ, gq), ("dK", dK, gk), ("dV", dV, gv)):
+            if not _close(a, r, 1e-9):
+                bad.append(f"{name} != torch autograd (case {seed})")
+        # invariants: sum over keys of dK is 0, sum over keys of dV = sum over queries of dO
+        if not _close(dK.sum(0), np.zeros((H, d)), 1e-9):
+            bad.append(f"sum of dK over keys is not 0 (case {seed})")
+        if not _close(dV.sum(0), do.sum(0), 1e-9):
+            bad.append(f"sum of dV over keys != sum of dO (case {seed})")
+    # central finite differences of L = <O, dO> against the oracle's own forward
+    q, k, v, do, bm = random_case(20, 7, 1, 3, 3, 0.6)
+    rp, ci = bitmap_to_csr(bm)
+    dQ, dK, dV = bsattn_bwd(q, k, v, do, rp, ci, 3)
+    eps = 1e-6
+
+    def loss(qq, kk, vv):
+        return float((bsattn_fwd(qq, kk, vv, rp, ci, 3)[0] * do).sum())
+
+    for name, which, grad in (("dQ", 0, dQ), ("dK", 1, dK), ("dV", 2, dV)):
+        fd = np.zeros_like(grad)
+        for pos in np.ndindex(grad.shape):
+            args_p = [q.copy(), k.copy(), v.copy()]
+            args_m = [q.copy(), k.copy(), v.copy()]
+            args_p[which][pos] += eps
+            args_m[which][pos] -= eps
+            fd[pos] = (loss(*args_p) - loss(*args_m)) / (2 * eps)
+        if not np.allclose(fd, grad, atol=1e-7, rtol=1e-6):
+            bad.append(f"{name} != finite differences")
+    return bad
+
+
+def check_subsample_consistency(o, bitmap_to_csr):
+    """Row-subset helpers agree with the full oracle functions."""
+    bad = []
+    q, k, v, do, bm = random_case(30, 21, 2, 4, 4, 0.5)
+    rp, ci = bitmap_to_csr(bm)
+    O, LSE = o.bsattn_fwd(q, k, v, rp, ci, 4)
+    dQ, dK, dV = o.bsattn_bwd(q, k, v, do, rp, ci, 4)
+    rows = np.array([0, 3, 4, 9, 20])
+    for h in range(2):
+        Or, Lr = o.bsattn_fwd_rows(q, k, v, rp, ci, 4, h, rows)
+        if not (_close(Or, O[rows, h]) and _close(Lr, LSE[h, rows])):
+            bad.append("bsattn_fwd_rows")
+        if not _close(o.bsattn_bwd_dq_rows(q, k, v, do, rp, ci, 4, h, rows), dQ[rows, h]):
+            bad.append("bsattn_bwd_dq_rows")
+        dk, dv = o.bsattn_bwd_dkdv_rows(q, k, v, do, rp, ci, 4, h, rows)
+        if not (_close(dk, dK[rows, h]) and _close(dv, dV[rows, h])):
+            bad.append("bsattn_bwd_dkdv_rows")
+    return bad

@@ -1,0 +1,197 @@
+"""Pins of the fp64 oracle (CPU only) and planted-mistake checks that show the pins bite."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle.ultratex_oracle as o
+import pins
+from synth import CONFIGS
+
+
+def test_compaction_and_scatter_pinned():
+    assert pins.check_compaction(o.fg_compact, o.fg_scatter) == []
+
+
+def test_block_lists_pinned():
+    assert pins.check_block_lists(o.bitmap_to_csr, o.csr_to_csc) == []
+
+
+def test_topk_pinned():
+    assert pins.check_topk(o.topk_block_mask, o.block_pool, o.k_rho) == []
+
+
+def test_forward_pinned():
+    assert pins.check_forward(o.bsattn_fwd, o.bitmap_to_csr) == []
+
+
+def test_backward_pinned():
+    assert pins.check_backward(o.bsattn_fwd, o.bsattn_bwd, o.bitmap_to_csr) == []
+
+
+def test_row_subset_helpers_agree():
+    assert pins.check_subsample_consistency(o, o.bitmap_to_csr) == []
+
+
+def test_canvas_arithmetic(golden_dir):
+    """Sec. 3.1 token counts and the Table S1 length column pin the canvas generator."""
+    with open(os.path.join(golden_dir, "token_counts.json")) as f:
+        g = json.load(f)
+    w = CONFIGS["c2048"]
+    assert w.tokens_per_image == g["tokens_per_image_2048"]
+    assert w.n_images == sum(g["images"].values())
+    assert w.T == g["canvas_tokens_2048"]
+    for f_str, length in g["table_s1_token_length"].items():
+        n = w.with_(fg_frac=float(f_str)).N
+        assert abs(n - (length - g["text_prefix_tokens_reading"])) <= 12, (f_str, n, length)
+
+
+def test_flop_count_matches_definition():
+    rp = np.array([0, 2, 3], np.int32)
+    ci = np.array([0, 1, 1], np.int32)
+    # N = 6, b = 4: tiles of 4 and 2 rows.  pairs (0,0):4*4, (0,1):4*2, (1,1):2*2
+    assert o.retained_flops_fwd(rp, ci, 6, 4, 8) == 4 * 8 * (16 + 8 + 4)
+
+
+# ------------------------------------------------------------ planted mistakes
+def _fwd_no_scale(q, k, v, rp, ci, b, scale=None):
+    return o.bsattn_fwd(q, k, v, rp, ci, b, 1.0 if scale is None else scale)
+
+
+def _fwd_transposed_lists(q, k, v, rp, ci, b, scale=None):
+    N, H, _ = q.shape
+    nq = o.n_blocks(N, b)
+    bm = o.csr_to_bitmap(rp, ci, H, nq, nq).transpose(0, 2, 1)
+    rp2, ci2 = o.bitmap_to_csr(np.ascontiguousarray(bm))
+    return o.bsattn_fwd(q, k, v, rp2, ci2, b, scale)
+
+
+def _fwd_drop_tail(q, k, v, rp, ci, b, scale=None):
+    N = q.shape[0]
+    O, L = o.bsattn_fwd(q, k, v, rp, ci, b, scale)
+    if N % b:
+        O[N - (N % b):] = 0
+    return O, L
+
+
+def _fwd_lse_log2(q, k, v, rp, ci, b, scale=None):
+    O, L = o.bsattn_fwd(q, k, v, rp, ci, b, scale)
+    return O, L / math.log(2)
+
+
+def _bwd_sign(q, k, v, do, rp, ci, b, scale=None):
+    dQ, dK, dV = o.bsattn_bwd(q, k, v, do, rp, ci, b, scale)
+    return -dQ, dK, dV
+
+
+def _bwd_no_D(q, k, v, do, rp, ci, b, scale=None):
+    # dS = P * dP, forgetting the D_r term
+    N, H, d = q.shape
+    scale = 1.0 / math.sqrt(d) if scale is None else scale
+    dQ, dK, dV = o.bsattn_bwd(q, k, v, do, rp, ci, b, scale)
+    nq = o.n_blocks(N, b)
+    for h in range(H):
+        for i in range(nq):
+            rows = o.tile_rows(i, N, b)
+            keys = o._keys(rp, ci, h * nq + i, N, b)
+            if len(keys) == 0:
+                continue
+            _, _, p = o._row_attention(q[rows, h], k[keys, h], v[keys, h], scale)
+            dS = p * (do[rows, h] @ v[keys, h].T)
+            dQ[rows, h] = (dS @ k[keys, h]) * scale
+    return dQ, dK, dV
+
+
+def _bwd_dv_transposed(q, k, v, do, rp, ci, b, scale=None):
+    dQ, dK, dV = o.bsattn_bwd(q, k, v, do, rp, ci, b, scale)
+    return dQ, dV, dK
+
+
+def _topk_smallest(qc, kc, b, rho):
+    return o.topk_block_mask(-qc, kc, b, rho)
+
+
+def _topk_tie_high(qc, kc, b, rho):
+    N, H, _ = qc.shape
+    nq = o.n_blocks(N, b)
+    kr = o.k_rho(rho, nq)
+    lists = []
+    for h in range(H):
+        sc = o.compressed_scores(qc[:, h], kc[:, h], b)
+        for i in range(nq):
+            order = np.lexsort((-np.arange(nq), -sc[i]))
+            lists.append(np.sort(order[:kr]))
+    return (np.arange(H * nq + 1) * kr).astype(np.int32), np.concatenate(lists).astype(np.int32), None, kr
+
+
+def _pool_sum(x, b):
+    x = np.asarray(x, np.float64)
+    return np.stack([x[o.tile_rows(i, x.shape[0], b)].sum(0) for i in range(o.n_blocks(x.shape[0], b))])
+
+
+def _topk_pool_sum(qc, kc, b, rho):
+    N, H, _ = qc.shape
+    nq = o.n_blocks(N, b)
+    kr = o.k_rho(rho, nq)
+    lists = []
+    for h in range(H):
+        sc = _pool_sum(qc[:, h], b) @ _pool_sum(kc[:, h], b).T
+        for i in range(nq):
+            lists.append(np.sort(np.lexsort((np.arange(nq), -sc[i]))[:kr]))
+    return (np.arange(H * nq + 1) * kr).astype(np.int32), np.concatenate(lists).astype(np.int32), None, kr
+
+
+def _krho_ceil(rho, nk):
+    return max(1, int(math.ceil(rho * nk)))
+
+
+def _topk_krho_ceil(qc, kc, b, rho):
+    N, H, _ = qc.shape
+    nq = o.n_blocks(N, b)
+    kr = _krho_ceil(rho, nq)
+    lists = []
+    for h in range(H):
+        sc = o.compressed_scores(qc[:, h], kc[:, h], b)
+        for i in range(nq):
+            lists.append(np.sort(np.lexsort((np.arange(nq), -sc[i]))[:kr]))
+    return (np.arange(H * nq + 1) * kr).astype(np.int32), np.concatenate(lists).astype(np.int32), None, kr
+
+
+def _compact_off_by_one(mask, xs):
+    idx, out = o.fg_compact(mask, xs)
+    idx = np.minimum(idx + 1, len(mask) - 1).astype(np.int32)
+    return idx, [np.asarray(x)[idx] for x in xs]
+
+
+def _scatter_zero_everything(idx, src, dst_in, mode=0, fill_row=None):
+    return o.fg_scatter(idx, src, dst_in, o.BG_ZERO, fill_row)
+
+
+def _csr_descending(bm):
+    rp, ci = o.bitmap_to_csr(bm)
+    ci = ci.copy()
+    for r in range(len(rp) - 1):
+        ci[rp[r]:rp[r + 1]] = ci[rp[r]:rp[r + 1]][::-1]
+    return rp, ci
+
+
+@pytest.mark.parametrize("name,check", [
+    ("fwd without 1/sqrt(d)", lambda: pins.check_forward(_fwd_no_scale, o.bitmap_to_csr)),
+    ("fwd with transposed block lists", lambda: pins.check_forward(_fwd_transposed_lists, o.bitmap_to_csr)),
+    ("fwd dropping the partial tile", lambda: pins.check_forward(_fwd_drop_tail, o.bitmap_to_csr)),
+    ("fwd LSE in log2", lambda: pins.check_forward(_fwd_lse_log2, o.bitmap_to_csr)),
+    ("bwd dQ sign", lambda: pins.check_backward(o.bsattn_fwd, _bwd_sign, o.bitmap_to_csr)),
+    ("bwd without the D term", lambda: pins.check_backward(o.bsattn_fwd, _bwd_no_D, o.bitmap_to_csr)),
+    ("bwd dK/dV swapped", lambda: pins.check_backward(o.bsattn_fwd, _bwd_dv_transposed, o.bitmap_to_csr)),
+    ("Top-K keeps smallest", lambda: pins.check_topk(_topk_smallest, o.block_pool, o.k_rho)),
+    ("Top-K tie toward larger index", lambda: pins.check_topk(_topk_tie_high, o.block_pool, o.k_rho)),
+    ("Top-K sum pooling", lambda: pins.check_topk(_topk_pool_sum, _pool_sum, o.k_rho)),
+    ("Top-K ceil(rho N_k)", lambda: pins.check_topk(_topk_krho_ceil, o.block_pool, _krho_ceil)),
+    ("compaction off by one", lambda: pins.check_compaction(_compact_off_by_one, o.fg_scatter)),
+    ("scatter ignores the mode", lambda: pins.check_compaction(o.fg_compact, _scatter_zero_everything)),
+    ("CSR lists descending", lambda: pins.check_block_lists(_csr_descending, o.csr_to_csc)),
+])
+def test_planted_mistake_is_caught(name, check):
+    assert check() != [], f"the pins did not catch: {name}"
