@@ -1,0 +1,178 @@
+/*
+ * ultratex.h -- C ABI of the foreground-only block-sparse attention path of
+ * "UltraTex: Unleashing 2K Multi-View Diffusion for 3D Texturing".
+ *
+ * The path (Sec. 3.2 and Sec. 3.3 of the paper):
+ *   1. ut_fg_compact  -- Background Token Dropping: gather the foreground
+ *                        tokens of the multi-view canvas (Gather_{M_fg}).
+ *   2. ut_block_mask  -- per head and query block, the list of key blocks to
+ *                        attend to: Top-K over mean-pooled compressed scores
+ *                        S_c = pool(Q) pool(K)^T, or a caller-given bitmap.
+ *   3. ut_bsattn_fwd  -- block-sparse attention over the listed key blocks.
+ *   4. ut_bsattn_bwd  -- its gradient (the paper trains stage 3 with it).
+ *   5. ut_fg_scatter  -- put compacted rows back at their canvas positions.
+ *
+ * Conventions shared by every entry point
+ *   - Pointers are DEVICE pointers unless the parameter name starts with h_
+ *     (host memory).  The caller owns every buffer, including workspaces
+ *     sized by the *_workspace_size functions.  No entry point allocates or
+ *     frees memory, synchronises the device or keeps global state.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy stream).  All
+ *     work is enqueued on it; results are valid once the stream has reached
+ *     the enqueued work.
+ *   - Argument errors are detected on the host BEFORE anything is enqueued
+ *     and returned as UT_ERR_INVALID_ARG / UT_ERR_UNSUPPORTED /
+ *     UT_ERR_CAPACITY; a failed launch returns UT_ERR_CUDA.
+ *   - Errors found on the device (a bounded wait that expired, a capacity
+ *     that only the device can see) are written into `dev_status`: one
+ *     int32 in device memory that the caller zeroes beforehand and reads
+ *     after synchronising.  The first error wins.  `dev_status` may be NULL
+ *     where noted.
+ *   - Token-major layout: a token row holds H heads of d elements each, head
+ *     h at element offset h*d; consecutive tokens are `row_stride` elements
+ *     apart.  Row starts must be 16-byte aligned.
+ */
+#ifndef ULTRATEX_H
+#define ULTRATEX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  UT_OK = 0,
+  UT_ERR_INVALID_ARG = 1,   /* null pointer, misalignment, negative size ... */
+  UT_ERR_UNSUPPORTED = 2,   /* a valid but unimplemented shape or dtype */
+  UT_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed */
+  UT_ERR_TIMEOUT = 4,       /* (device) a bounded wait expired; kernel gave up */
+  UT_ERR_CAPACITY = 5       /* an output buffer is too small */
+} ut_status;
+
+typedef enum { UT_BF16 = 0, UT_F32 = 1 } ut_dtype;
+
+/* Background handling of ut_fg_scatter. */
+enum { UT_BG_KEEP = 0, UT_BG_ZERO = 1, UT_BG_FILL = 2 };
+/* Modes of ut_block_mask. */
+enum { UT_MASK_TOPK = 0, UT_MASK_BITMAP = 1 };
+
+/* Shape of the compacted attention problem.  Sec. 3.3 states it per head as
+ * Q, K, V in R^{N x d} partitioned into blocks of b_q and b_kv rows; here
+ * b_q = b_kv = block.  N_q = N_k = ceil(N / block); the last block may be
+ * partial (its missing key rows are excluded, its missing query rows are not
+ * written). */
+typedef struct {
+  int64_t n_tokens;    /* N: rows of the compacted sequence, >= 0 */
+  int32_t n_heads;     /* H >= 1 */
+  int32_t head_dim;    /* d: 64 or 128 */
+  int32_t block;       /* b: bf16 tensor-core path 128; fp32 path 32, 64, 128 */
+  int32_t dtype;       /* ut_dtype of Q, K, V, O, dO, dQ, dK, dV */
+  int64_t row_stride;  /* elements between consecutive tokens, >= H*d, multiple of 8 */
+} ut_attn_shape;
+
+const char* ut_strerror(ut_status s);
+
+/* K_rho = max(1, floor(rho * n_k)) evaluated in double precision
+ * (Sec. 3.3, the Top-K retention count). */
+int32_t ut_topk_count(double rho, int64_t n_k);
+
+/* ------------------------------------------------------------------------
+ * Background Token Dropping (Sec. 3.2: z~ = Gather_{M_fg}(z); retained tokens
+ * are concatenated in canvas order and keep their canvas position, which is
+ * their RoPE index).
+ *
+ *   mask      [T] uint8, nonzero = foreground.
+ *   h_src     host array of n_tensors device pointers, each [T rows x row_bytes].
+ *   h_dst     host array of n_tensors device pointers, each [capacity rows x row_bytes].
+ *   row_bytes bytes per token row (multiple of 16; pointers 16-byte aligned).
+ *   capacity  rows available in each dst and in idx_out.
+ *   idx_out   [capacity] int32: canvas position of compacted row n, ascending.
+ *   n_out     one int32 (device): N = number of foreground tokens.
+ *   ws        workspace of ut_fg_compact_workspace_size(T) bytes.
+ *   dev_status (may be NULL) receives UT_ERR_CAPACITY when N > capacity; rows
+ *             beyond capacity are then not written (n_out still holds N).
+ * 1 <= n_tensors <= 8; T may be 0 (then N = 0).  Gathering reuses nothing
+ * from a previous call. */
+size_t ut_fg_compact_workspace_size(int64_t T);
+ut_status ut_fg_compact(const uint8_t* mask, int64_t T, int32_t n_tensors,
+                        const void* const* h_src, void* const* h_dst, int64_t row_bytes,
+                        int64_t capacity, int32_t* idx_out, int32_t* n_out,
+                        void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Scatter compacted rows back to the canvas: dst[idx[n]] = src[n] for n < N.
+ * Background rows (canvas positions not in idx) are, by bg_mode:
+ *   UT_BG_KEEP  not written ("background positions are not updated", Sec. 3.2);
+ *   UT_BG_ZERO  set to zero (the adjoint of the gather, for gradients);
+ *   UT_BG_FILL  set to fill_row (row_bytes bytes, device), the canonical
+ *               background latent of Sec. 3.4's z_mix.
+ * idx must be strictly increasing and < T (as ut_fg_compact writes it).
+ * n is the host-side N; T the canvas rows of each dst. */
+ut_status ut_fg_scatter(const int32_t* idx, int64_t n, int32_t n_tensors,
+                        const void* const* h_src, void* const* h_dst, int64_t row_bytes,
+                        int32_t bg_mode, const void* fill_row, int64_t T, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Block mask M_c as per-(head, query block) key-block lists (Sec. 3.3).
+ * Rows r = h*N_q + i (head-major).  Lists are ascending.
+ *
+ * UT_MASK_TOPK: S_c = pool(Q) pool(K)^T per head with mean pooling over the
+ *   valid rows of each block (fp32), then per row the K_rho =
+ *   ut_topk_count(rho, N_k) largest scores; equal scores go to the smaller
+ *   key-block index.  `q`, `k` are the compacted [N, H, d] tensors; `bitmap`
+ *   is ignored.  row_ptr[r] = r * K_rho.
+ * UT_MASK_BITMAP: `bitmap` is [H, N_q, N_k] uint8 (nonzero = keep), given by
+ *   the caller (structured masks); `q`, `k`, `rho` are ignored.  A row may be
+ *   empty; the attention then writes O = 0 and LSE = -inf for it.
+ *
+ *   row_ptr   [H*N_q + 1] int32, col_idx [col_cap] int32 (CSR).
+ *   col_ptr_t [H*N_k + 1] int32, row_idx_t [col_cap] int32: the transpose
+ *             (per key block, ascending query blocks) for the backward; pass
+ *             both NULL to skip it.
+ *   ws        ut_block_mask_workspace_size(shape, mode) bytes.
+ *   dev_status receives UT_ERR_CAPACITY if the bitmap holds more than
+ *             col_cap entries (must be non-NULL in bitmap mode).
+ * TOPK mode checks H*N_q*K_rho <= col_cap on the host. */
+size_t ut_block_mask_workspace_size(const ut_attn_shape* shape, int32_t mode);
+ut_status ut_block_mask(const ut_attn_shape* shape, int32_t mode,
+                        const void* q, const void* k, double rho, const uint8_t* bitmap,
+                        int32_t* row_ptr, int32_t* col_idx, int64_t col_cap,
+                        int32_t* col_ptr_t, int32_t* row_idx_t,
+                        void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Block-sparse attention forward (Sec. 3.3):
+ *   O_i = softmax(Q_i K_{S_i}^T * softmax_scale) V_{S_i}
+ * for every head and query block i, S_i the list row_ptr/col_idx gives.
+ *   q, k, v, o  [N, H, d] token-major with shape->row_stride (dtype of shape).
+ *   lse         [H, N] fp32 natural-log row normalisers (m + log sum exp).
+ *   softmax_scale  1/sqrt(d) in the paper; any positive value accepted.
+ * bf16 runs on the tcgen05 tensor cores (fp32 accumulation, P rounded to
+ * bf16 before P V, O rounded to bf16); fp32 runs a CUDA-core fp32 kernel. */
+ut_status ut_bsattn_fwd(const ut_attn_shape* shape, const void* q, const void* k, const void* v,
+                        const int32_t* row_ptr, const int32_t* col_idx, float softmax_scale,
+                        void* o, float* lse, int32_t* dev_status, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Gradient of ut_bsattn_fwd with respect to Q, K, V given dO:
+ *   D_r = dO_r . O_r,  P = exp(S - LSE),  dV = P^T dO,  dS = P o (dO V^T - D),
+ *   dQ = dS K * scale,  dK = dS^T Q * scale
+ * over the retained block pairs only.  Needs the CSR lists and their
+ * transpose (col_ptr_t / row_idx_t from ut_block_mask).
+ *   o, lse      the forward's outputs.
+ *   dq, dk, dv  [N, H, d] outputs (dtype of shape), fully overwritten.
+ *   ws          ut_bsattn_bwd_workspace_size(shape) bytes. */
+size_t ut_bsattn_bwd_workspace_size(const ut_attn_shape* shape);
+ut_status ut_bsattn_bwd(const ut_attn_shape* shape, const void* q, const void* k, const void* v,
+                        const void* o, const float* lse, const void* dout,
+                        const int32_t* row_ptr, const int32_t* col_idx,
+                        const int32_t* col_ptr_t, const int32_t* row_idx_t, float softmax_scale,
+                        void* dq, void* dk, void* dv, void* ws, size_t ws_bytes,
+                        int32_t* dev_status, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ULTRATEX_H */

@@ -1,0 +1,384 @@
+// Block-sparse attention forward on the 5th-generation tensor cores (Sec. 3.3):
+//   O_i = softmax(Q_i K_{S_i}^T * scale) V_{S_i}
+// for every (head, query block i), iterating only the listed key blocks.
+//
+// Persistent kernel, one CTA per SM, work items (h, i) in head-major order so
+// that the CTAs in flight share one head's K/V in L2.  Roles (192 threads):
+//   warp 0      TMA producer: Q tile of the item, then K_j / V_j of every
+//               listed key block into a 2-stage ring (128B-swizzled tiles).
+//   warp 1      TMEM owner and MMA issuer (one elected thread):
+//               S_t = Q K_t^T into one of two TMEM S buffers, then
+//               O += P_{t-1} V_{t-1} into the TMEM O accumulator.
+//   warps 2-5   softmax: thread = query row = TMEM lane.  Reads S_t from TMEM,
+//               masks the ragged last key block, keeps a running row maximum
+//               (rescaling O in TMEM only when the maximum grew by more than
+//               2^8, so the exponentials stay bounded), writes P_t as bf16 into
+//               a 128B-swizzled shared tile for the P V MMA, and finally
+//               normalises O, writes O (bf16) and LSE (fp32, natural log).
+// TMEM: S buffers at columns [0,128) and [128,256), O at [256, 256+D).
+// Every wait is bounded; on expiry the kernel records UT_ERR_TIMEOUT,
+// drains its own copies and MMAs, frees TMEM and returns.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace ut {
+
+constexpr int kBM = 128;  // query rows per tile
+constexpr int kBN = 128;  // key rows per tile
+constexpr int kFwdThreads = 192;
+constexpr uint32_t kTileChunkBytes = 128 * 128;  // 128 rows x 128 bytes (64 bf16)
+
+template <int D>
+struct FwdSmem {
+  static constexpr int kChunks = D / 64;
+  static constexpr uint32_t kQBytes = kBM * D * 2;
+  static constexpr uint32_t kKVBytes = kBN * D * 2;
+  static constexpr uint32_t kPBytes = kBM * kBN * 2;
+  alignas(1024) uint8_t q[kQBytes];
+  alignas(1024) uint8_t k[2][kKVBytes];
+  alignas(1024) uint8_t v[2][kKVBytes];
+  alignas(1024) uint8_t p[2][kPBytes];
+  uint64_t q_full, q_empty;
+  uint64_t k_full[2], v_full[2], kv_empty[2];
+  uint64_t s_full[2], s_empty[2];
+  uint64_t p_full[2], pv_done[2];
+  uint64_t o_empty, mma_done;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+struct FwdParams {
+  const int32_t* row_ptr;
+  const int32_t* col_idx;
+  __nv_bfloat16* o;
+  float* lse;
+  int32_t* status;
+  int64_t N;
+  int64_t rs;  // elements between tokens
+  int H, nq;
+  int n_items;
+  float scale_log2;  // softmax scale * log2(e)
+  uint64_t timeout_ns;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kFwdThreads, 1)
+    attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                       const __grid_constant__ CUtensorMap tm_v, const FwdParams prm) {
+  extern __shared__ uint8_t smem_raw[];
+  FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  constexpr int C = FwdSmem<D>::kChunks;
+  const uint32_t warp = warp_id();
+  const uint32_t lane = lane_id();
+  volatile int* abort_flag = &sm.abort_flag;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&sm.q_full, 1);
+    mbar_init(&sm.q_empty, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.k_full[s], 1);
+      mbar_init(&sm.v_full[s], 1);
+      mbar_init(&sm.kv_empty[s], 1);
+      mbar_init(&sm.s_full[s], 1);
+      mbar_init(&sm.s_empty[s], 4);
+      mbar_init(&sm.p_full[s], 4);
+      mbar_init(&sm.pv_done[s], 1);
+    }
+    mbar_init(&sm.o_empty, 4);
+    mbar_init(&sm.mma_done, 1);
+    sm.abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+
+  const int G = gridDim.x;
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      const uint64_t pol_kv = policy_evict_last();
+      const uint64_t pol_q = policy_evict_first();
+      uint32_t qi = 0, kv = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+        const int h = w / prm.nq, i = w % prm.nq;
+        const int beg = prm.row_ptr[w], L = prm.row_ptr[w + 1] - beg;
+        if (L <= 0) continue;
+        if (!(ok = mbar_wait(&sm.q_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        mbar_expect_tx(&sm.q_full, FwdSmem<D>::kQBytes);
+        for (int c = 0; c < C; ++c)
+          tma_load_2d(sm.q + c * kTileChunkBytes, &tm_q, &sm.q_full, h * D + c * 64, i * kBM, pol_q);
+        ++qi;
+        for (int t = 0; t < L; ++t, ++kv) {
+          const int j = prm.col_idx[beg + t];
+          const int st = kv & 1;
+          const uint32_t n = kv >> 1;
+          if (!(ok = mbar_wait(&sm.kv_empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&sm.k_full[st], FwdSmem<D>::kKVBytes);
+          for (int c = 0; c < C; ++c)
+            tma_load_2d(sm.k[st] + c * kTileChunkBytes, &tm_k, &sm.k_full[st], h * D + c * 64, j * kBN, pol_kv);
+          mbar_expect_tx(&sm.v_full[st], FwdSmem<D>::kKVBytes);
+          for (int c = 0; c < C; ++c)
+            tma_load_2d(sm.v[st] + c * kTileChunkBytes, &tm_v, &sm.v_full[st], h * D + c * 64, j * kBN, pol_kv);
+        }
+      }
+      // Drain: every issued copy has landed before the CTA may exit.
+      const uint64_t t0 = globaltimer();
+      auto drain = [&](uint64_t* bar, uint32_t parity) {
+        while (!mbar_try_wait(bar, parity))
+          if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+      };
+      if (qi > 0) drain(&sm.q_full, (qi - 1) & 1);
+      for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) {
+        drain(&sm.k_full[u & 1], (u >> 1) & 1);
+        drain(&sm.v_full[u & 1], (u >> 1) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN, false, false);
+      constexpr uint32_t idesc_o = idesc_bf16_f32(kBM, D, false, true);
+      const uint32_t q_addr = smem_u32(sm.q);
+      uint32_t qi = 0, oi = 0, kv0 = 0, sc0 = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+        const int L = prm.row_ptr[w + 1] - prm.row_ptr[w];
+        if (L <= 0) continue;
+        if (!(ok = mbar_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        for (int t = 0; t <= L && ok; ++t) {
+          if (t < L) {
+            const uint32_t kv = kv0 + t, st = kv & 1, n = kv >> 1;
+            const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
+            if (!(ok = mbar_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.s_empty[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+            const uint32_t k_addr = smem_u32(sm.k[st]);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kTileChunkBytes + (kk & 3) * 32;
+              mma_bf16_ss(tmem + sb * 128, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024),
+                          idesc_s, kk > 0);
+            }
+            mma_commit(&sm.s_full[sb]);
+            if (t == L - 1) mma_commit(&sm.q_empty);
+          }
+          if (t >= 1) {
+            const uint32_t u = t - 1;
+            const uint32_t kv = kv0 + u, st = kv & 1, n = kv >> 1;
+            const uint32_t sc = sc0 + u, pb = sc & 1, np = sc >> 1;
+            if (!(ok = mbar_wait(&sm.p_full[pb], np & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (u == 0 && !(ok = mbar_wait(&sm.o_empty, (oi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+              break;
+            tc_fence_after();
+            const uint32_t p_addr = smem_u32(sm.p[pb]);
+            const uint32_t v_addr = smem_u32(sm.v[st]);
+#pragma unroll
+            for (int kk = 0; kk < kBN / 16; ++kk) {
+              const uint32_t aoff = (kk >> 2) * kTileChunkBytes + (kk & 3) * 32;
+              mma_bf16_ss(tmem + 256, sdesc_sw128(p_addr + aoff, 16, 1024),
+                          sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024), idesc_o, (u > 0 || kk > 0));
+            }
+            mma_commit(&sm.pv_done[pb]);
+            mma_commit(&sm.kv_empty[st]);
+          }
+        }
+        kv0 += L;
+        sc0 += L;
+        ++qi;
+        ++oi;
+      }
+      // Drain: all MMAs issued by this thread complete before TMEM is freed.
+      mma_commit(&sm.mma_done);
+      const uint64_t t0 = globaltimer();
+      while (!mbar_try_wait(&sm.mma_done, 0))
+        if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+    }
+  } else {
+    // ------------------------------------------------------------- softmax
+    const uint32_t quarter = warp & 3;
+    const uint32_t row = quarter * 32 + lane;
+    const uint32_t lane_base = (quarter * 32) << 16;
+    const float c = prm.scale_log2;
+    uint32_t sc0 = 0;
+    bool ok = true;
+    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+      const int h = w / prm.nq, i = w % prm.nq;
+      const int beg = prm.row_ptr[w], L = prm.row_ptr[w + 1] - beg;
+      const int64_t grow = (int64_t)i * kBM + row;
+      const bool row_ok = grow < prm.N;
+      __nv_bfloat16* orow = prm.o + grow * prm.rs + (int64_t)h * D;
+      if (L <= 0) {
+        if (row_ok) {
+          for (int e = 0; e < D; e += 8) *reinterpret_cast<uint4*>(orow + e) = make_uint4(0, 0, 0, 0);
+          prm.lse[(int64_t)h * prm.N + grow] = -INFINITY;
+        }
+        continue;
+      }
+      float m_used = 0.f, l = 0.f;
+      for (int t = 0; t < L; ++t) {
+        const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
+        if (!(ok = warp_wait(&sm.s_full[sb], ns & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
+        float s[kBN];
+#pragma unroll
+        for (int g = 0; g < kBN / 32; ++g) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + sb * 128 + g * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int x = 0; x < 32; ++x) s[g * 32 + x] = __uint_as_float(r[x]);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.s_empty[sb]);
+        // ragged last key block: columns past N do not exist
+        const int j = prm.col_idx[beg + t];
+        const int64_t nv = prm.N - (int64_t)j * kBN;
+        if (nv < kBN) {
+#pragma unroll
+          for (int x = 0; x < kBN; ++x)
+            if (x >= nv) s[x] = -INFINITY;
+        }
+        float mx = s[0];
+#pragma unroll
+        for (int x = 1; x < kBN; ++x) mx = fmaxf(mx, s[x]);
+        mx *= c;
+        if (t == 0) {
+          m_used = mx;
+        } else {
+          const bool need = mx > m_used + 8.0f;
+          if (__any_sync(0xffffffffu, need)) {
+            const uint32_t pc = sc - 1;
+            if (!(ok = warp_wait(&sm.pv_done[pc & 1], (pc >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
+              break;
+            tc_fence_after();
+            const float alpha = need ? ex2_approx(m_used - mx) : 1.0f;
+#pragma unroll
+            for (int g = 0; g < D / 32; ++g) {
+              uint32_t r[32];
+              tmem_ld32(tmem + lane_base + 256 + g * 32, r);
+              tmem_wait_ld();
+#pragma unroll
+              for (int x = 0; x < 32; ++x) r[x] = __float_as_uint(__uint_as_float(r[x]) * alpha);
+              tmem_st32(tmem + lane_base + 256 + g * 32, r);
+            }
+            tmem_wait_st();
+            if (need) {
+              l *= alpha;
+              m_used = mx;
+            }
+          }
+        }
+        // P = exp2(s * c - m_used), rounded to bf16 for the P V MMA
+        uint32_t pk[kBN / 2];
+        float lsum = 0.f;
+#pragma unroll
+        for (int x = 0; x < kBN; x += 2) {
+          const float p0 = ex2_approx(fmaf(s[x], c, -m_used));
+          const float p1 = ex2_approx(fmaf(s[x + 1], c, -m_used));
+          lsum += p0 + p1;
+          pk[x / 2] = pack_bf16x2(p0, p1);
+        }
+        l += lsum;
+        // the P buffer is free once the P V MMA of its previous use finished
+        if (!(ok = warp_wait(&sm.pv_done[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        const uint32_t p_row = smem_u32(sm.p[sb]) + row * 128;
+#pragma unroll
+        for (int u = 0; u < kBN / 8; ++u) {
+          const uint32_t chunk = u >> 3, unit = u & 7;
+          const uint32_t addr = p_row + chunk * kTileChunkBytes + ((unit ^ (row & 7)) << 4);
+          st_shared_v4(addr, pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.p_full[sb]);
+      }
+      if (!ok) break;
+      // epilogue: O / l -> bf16, LSE
+      const uint32_t last = sc0 + L - 1;
+      if (!(ok = warp_wait(&sm.pv_done[last & 1], (last >> 1) & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+      tc_fence_after();
+      const float inv = 1.0f / l;
+#pragma unroll
+      for (int g = 0; g < D / 32; ++g) {
+        uint32_t r[32];
+        tmem_ld32(tmem + lane_base + 256 + g * 32, r);
+        tmem_wait_ld();
+        if (row_ok) {
+#pragma unroll
+          for (int x = 0; x < 32; x += 8) {
+            uint4 v;
+            v.x = pack_bf16x2(__uint_as_float(r[x + 0]) * inv, __uint_as_float(r[x + 1]) * inv);
+            v.y = pack_bf16x2(__uint_as_float(r[x + 2]) * inv, __uint_as_float(r[x + 3]) * inv);
+            v.z = pack_bf16x2(__uint_as_float(r[x + 4]) * inv, __uint_as_float(r[x + 5]) * inv);
+            v.w = pack_bf16x2(__uint_as_float(r[x + 6]) * inv, __uint_as_float(r[x + 7]) * inv);
+            *reinterpret_cast<uint4*>(orow + g * 32 + x) = v;
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.o_empty);
+      if (row_ok) prm.lse[(int64_t)h * prm.N + grow] = (m_used + log2f(l)) * 0.69314718055994531f;
+      sc0 += L;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+template <int D>
+static cudaError_t launch_d(const AttnProblem& p, const CUtensorMap& tq, const CUtensorMap& tk,
+                            const CUtensorMap& tv, const FwdParams& prm, int grid, cudaStream_t stream) {
+  const size_t smem = sizeof(FwdSmem<D>) + 1024;
+  cudaError_t e = cudaFuncSetAttribute(attn_fwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  attn_fwd_tc_kernel<D><<<grid, kFwdThreads, smem, stream>>>(tq, tk, tv, prm);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* k, const void* v,
+                               const int32_t* row_ptr, const int32_t* col_idx, void* o, float* lse, int32_t* status,
+                               uint64_t timeout_ns, int sms, cudaStream_t stream) {
+  const int n_items = p.H * p.nq;
+  if (n_items == 0) return cudaSuccess;
+  CUtensorMap tq, tk, tv;
+  const uint64_t inner = (uint64_t)p.H * p.d;
+  const uint64_t stride = (uint64_t)p.row_stride * 2;
+  if (!encode_tmap_2d_bf16(&tq, q, inner, p.N, stride, 64, kBM) ||
+      !encode_tmap_2d_bf16(&tk, k, inner, p.N, stride, 64, kBN) ||
+      !encode_tmap_2d_bf16(&tv, v, inner, p.N, stride, 64, kBN))
+    return cudaErrorInvalidValue;
+  FwdParams prm{};
+  prm.row_ptr = row_ptr;
+  prm.col_idx = col_idx;
+  prm.o = static_cast<__nv_bfloat16*>(o);
+  prm.lse = lse;
+  prm.status = status;
+  prm.N = p.N;
+  prm.rs = p.row_stride;
+  prm.H = p.H;
+  prm.nq = p.nq;
+  prm.n_items = n_items;
+  prm.scale_log2 = p.scale * 1.4426950408889634f;
+  prm.timeout_ns = timeout_ns;
+  const int grid = n_items < sms ? n_items : sms;
+  return p.d == 64 ? launch_d<64>(p, tq, tk, tv, prm, grid, stream) : launch_d<128>(p, tq, tk, tv, prm, grid, stream);
+}
+
+}  // namespace ut

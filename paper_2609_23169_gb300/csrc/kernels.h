@@ -1,0 +1,62 @@
+// Host-side launchers implemented by the .cu files; api.cu validates
+// arguments and calls these.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ut {
+
+// compact.cu
+size_t fg_compact_ws(int64_t T);
+cudaError_t launch_fg_compact(const uint8_t* mask, int64_t T, int n_tensors, const void* const* src,
+                              void* const* dst, int64_t row_bytes, int64_t capacity, int32_t* idx, int32_t* n_out,
+                              void* ws, int32_t* status, int sms, cudaStream_t stream);
+cudaError_t launch_fg_scatter(const int32_t* idx, int64_t N, int n_tensors, const void* const* src, void* const* dst,
+                              int64_t row_bytes, int bg_mode, const void* fill, int64_t T, int sms,
+                              cudaStream_t stream);
+
+// blockmask.cu
+struct MaskProblem {
+  int64_t N;
+  int H, d, block, dtype;
+  int64_t row_stride;
+  int nq;  // = nk
+};
+size_t block_mask_ws(const MaskProblem& p, int mode);
+cudaError_t launch_block_mask_topk(const MaskProblem& p, const void* q, const void* k, int k_rho, int32_t* row_ptr,
+                                   int32_t* col_idx, int32_t* col_ptr_t, int32_t* row_idx_t, int64_t col_cap,
+                                   void* ws, int32_t* status, int sms, cudaStream_t stream);
+cudaError_t launch_block_mask_bitmap(const MaskProblem& p, const uint8_t* bitmap, int32_t* row_ptr, int32_t* col_idx,
+                                     int32_t* col_ptr_t, int32_t* row_idx_t, int64_t col_cap, void* ws,
+                                     int32_t* status, cudaStream_t stream);
+
+// attention problems
+struct AttnProblem {
+  int64_t N;
+  int H, d, block, dtype;
+  int64_t row_stride;
+  int nq;
+  float scale;
+};
+
+// attn_simt.cu (fp32 path and the generic CUDA-core backward)
+cudaError_t launch_attn_fwd_simt(const AttnProblem& p, const void* q, const void* k, const void* v,
+                                 const int32_t* row_ptr, const int32_t* col_idx, void* o, float* lse,
+                                 cudaStream_t stream);
+size_t attn_bwd_simt_ws(const AttnProblem& p);
+cudaError_t launch_attn_bwd_simt(const AttnProblem& p, const void* q, const void* k, const void* v, const void* o,
+                                 const float* lse, const void* dout, const int32_t* row_ptr, const int32_t* col_idx,
+                                 const int32_t* col_ptr_t, const int32_t* row_idx_t, void* dq, void* dk, void* dv,
+                                 void* ws, cudaStream_t stream);
+
+// attn_fwd_tc.cu (bf16 tcgen05 forward)
+cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* k, const void* v,
+                               const int32_t* row_ptr, const int32_t* col_idx, void* o, float* lse, int32_t* status,
+                               uint64_t timeout_ns, int sms, cudaStream_t stream);
+
+// tensor maps (api.cu)
+bool encode_tmap_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner_elems, uint64_t rows,
+                         uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows);
+
+}  // namespace ut

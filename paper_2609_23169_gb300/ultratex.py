@@ -1,0 +1,227 @@
+"""Python binding of libultratex.so (ctypes; argument marshalling only).
+
+Every function here has the name of the C entry point it wraps and does
+nothing but check Python-side arguments, allocate outputs with torch when the
+caller did not pass them, and call the library on the current CUDA stream.
+There is no fallback: if the library is missing or a call fails, it raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "lib", "libultratex.so")
+
+UT_OK, UT_ERR_INVALID_ARG, UT_ERR_UNSUPPORTED, UT_ERR_CUDA, UT_ERR_TIMEOUT, UT_ERR_CAPACITY = range(6)
+UT_BF16, UT_F32 = 0, 1
+UT_BG_KEEP, UT_BG_ZERO, UT_BG_FILL = 0, 1, 2
+UT_MASK_TOPK, UT_MASK_BITMAP = 0, 1
+
+EXPORTS = (
+    "ut_strerror", "ut_topk_count", "ut_fg_compact_workspace_size", "ut_fg_compact", "ut_fg_scatter",
+    "ut_block_mask_workspace_size", "ut_block_mask", "ut_bsattn_fwd", "ut_bsattn_bwd_workspace_size",
+    "ut_bsattn_bwd",
+)
+
+
+class UtError(RuntimeError):
+    def __init__(self, fn: str, status: int, msg: str):
+        super().__init__(f"{fn} failed: {msg} (status {status})")
+        self.status = status
+
+
+class AttnShape(ctypes.Structure):
+    _fields_ = [("n_tokens", ctypes.c_int64), ("n_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("block", ctypes.c_int32), ("dtype", ctypes.c_int32), ("row_stride", ctypes.c_int64)]
+
+
+_lib = None
+_vp, _i32, _i64, _sz, _dbl, _flt = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t,
+                                     ctypes.c_double, ctypes.c_float)
+_ptrs = ctypes.POINTER(ctypes.c_void_p)
+
+
+def lib() -> ctypes.CDLL:
+    """Load libultratex.so (built by __graft_entry__.build()); raise if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+    L = ctypes.CDLL(LIB_PATH)
+    L.ut_strerror.restype = ctypes.c_char_p
+    L.ut_strerror.argtypes = [_i32]
+    L.ut_topk_count.restype = _i32
+    L.ut_topk_count.argtypes = [_dbl, _i64]
+    L.ut_fg_compact_workspace_size.restype = _sz
+    L.ut_fg_compact_workspace_size.argtypes = [_i64]
+    L.ut_fg_compact.restype = _i32
+    L.ut_fg_compact.argtypes = [_vp, _i64, _i32, _ptrs, _ptrs, _i64, _i64, _vp, _vp, _vp, _sz, _vp, _vp]
+    L.ut_fg_scatter.restype = _i32
+    L.ut_fg_scatter.argtypes = [_vp, _i64, _i32, _ptrs, _ptrs, _i64, _i32, _vp, _i64, _vp]
+    L.ut_block_mask_workspace_size.restype = _sz
+    L.ut_block_mask_workspace_size.argtypes = [ctypes.POINTER(AttnShape), _i32]
+    L.ut_block_mask.restype = _i32
+    L.ut_block_mask.argtypes = [ctypes.POINTER(AttnShape), _i32, _vp, _vp, _dbl, _vp, _vp, _vp, _i64, _vp, _vp,
+                                _vp, _sz, _vp, _vp]
+    L.ut_bsattn_fwd.restype = _i32
+    L.ut_bsattn_fwd.argtypes = [ctypes.POINTER(AttnShape), _vp, _vp, _vp, _vp, _vp, _flt, _vp, _vp, _vp, _vp]
+    L.ut_bsattn_bwd_workspace_size.restype = _sz
+    L.ut_bsattn_bwd_workspace_size.argtypes = [ctypes.POINTER(AttnShape)]
+    L.ut_bsattn_bwd.restype = _i32
+    L.ut_bsattn_bwd.argtypes = [ctypes.POINTER(AttnShape), _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _flt,
+                                _vp, _vp, _vp, _vp, _sz, _vp, _vp]
+    _lib = L
+    return L
+
+
+def _check(fn: str, st: int) -> None:
+    if st != UT_OK:
+        raise UtError(fn, st, lib().ut_strerror(st).decode())
+
+
+def _p(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream() -> int:
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _ptr_array(ts: Sequence[torch.Tensor]):
+    return (ctypes.c_void_p * len(ts))(*[t.data_ptr() for t in ts])
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return UT_BF16
+    if t.dtype == torch.float32:
+        return UT_F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def attn_shape(x: torch.Tensor, block: int) -> AttnShape:
+    """Shape of a token-major [N, H, d] tensor (rows may be padded: stride(0) >= H*d)."""
+    N, H, d = x.shape
+    assert x.stride(2) == 1 and x.stride(1) == d, "heads must be contiguous within a token row"
+    return AttnShape(N, H, d, block, _dtype_code(x), x.stride(0))
+
+
+def status_word(device=None) -> torch.Tensor:
+    return torch.zeros(1, dtype=torch.int32, device=device or "cuda")
+
+
+def check_status(st: torch.Tensor) -> None:
+    v = int(st.item())
+    if v != UT_OK:
+        raise UtError("device", v, lib().ut_strerror(v).decode())
+
+
+# ----------------------------------------------------------------- entry points
+def ut_topk_count(rho: float, n_k: int) -> int:
+    return int(lib().ut_topk_count(float(rho), int(n_k)))
+
+
+def ut_fg_compact(mask: torch.Tensor, srcs: Sequence[torch.Tensor], capacity: Optional[int] = None,
+                  outs: Optional[Sequence[torch.Tensor]] = None, idx: Optional[torch.Tensor] = None,
+                  n_out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                  status: Optional[torch.Tensor] = None):
+    """Background Token Dropping.  Returns (idx [capacity] i32, n_out [1] i32, outs)."""
+    T = mask.shape[0]
+    row_bytes = srcs[0][0].numel() * srcs[0].element_size() if T else 16
+    cap = T if capacity is None else int(capacity)
+    dev = mask.device
+    if outs is None:
+        outs = [torch.empty((cap,) + tuple(s.shape[1:]), dtype=s.dtype, device=dev) for s in srcs]
+    if idx is None:
+        idx = torch.empty(max(cap, 1), dtype=torch.int32, device=dev)
+    if n_out is None:
+        n_out = torch.empty(1, dtype=torch.int32, device=dev)
+    L = lib()
+    wsb = L.ut_fg_compact_workspace_size(T)
+    if ws is None:
+        ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device=dev)
+    st = L.ut_fg_compact(_p(mask), T, len(srcs), _ptr_array(srcs), _ptr_array(outs), row_bytes, cap, _p(idx),
+                         _p(n_out), _p(ws), ws.numel(), _p(status), _stream())
+    _check("ut_fg_compact", st)
+    return idx, n_out, list(outs)
+
+
+def ut_fg_scatter(idx: torch.Tensor, n: int, srcs: Sequence[torch.Tensor], dsts: Sequence[torch.Tensor],
+                  bg_mode: int = UT_BG_KEEP, fill_row: Optional[torch.Tensor] = None) -> None:
+    """dst[idx[i]] = src[i] for i < n; background rows per bg_mode."""
+    T = dsts[0].shape[0]
+    row_bytes = dsts[0][0].numel() * dsts[0].element_size()
+    st = lib().ut_fg_scatter(_p(idx), int(n), len(srcs), _ptr_array(srcs), _ptr_array(dsts), row_bytes, bg_mode,
+                             _p(fill_row), T, _stream())
+    _check("ut_fg_scatter", st)
+
+
+def ut_block_mask(shape: AttnShape, mode: int, q: Optional[torch.Tensor] = None, k: Optional[torch.Tensor] = None,
+                  rho: float = 0.0, bitmap: Optional[torch.Tensor] = None, col_cap: Optional[int] = None,
+                  with_transpose: bool = True, status: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                  out: Optional[tuple] = None):
+    """Key-block lists.  Returns (row_ptr, col_idx, col_ptr_t, row_idx_t) (the last two None if not asked)."""
+    nq = -(-shape.n_tokens // shape.block)
+    H = shape.n_heads
+    dev = (q if q is not None else bitmap).device
+    L = lib()
+    if col_cap is None:
+        col_cap = H * nq * (ut_topk_count(rho, nq) if mode == UT_MASK_TOPK else nq)
+    if out is None:
+        row_ptr = torch.empty(H * nq + 1, dtype=torch.int32, device=dev)
+        col_idx = torch.empty(max(col_cap, 1), dtype=torch.int32, device=dev)
+        col_ptr = torch.empty(H * nq + 1, dtype=torch.int32, device=dev) if with_transpose else None
+        row_idx = torch.empty(max(col_cap, 1), dtype=torch.int32, device=dev) if with_transpose else None
+    else:
+        row_ptr, col_idx, col_ptr, row_idx = out
+    wsb = L.ut_block_mask_workspace_size(ctypes.byref(shape), mode)
+    if ws is None:
+        ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device=dev)
+    if status is None and mode == UT_MASK_BITMAP:
+        status = status_word(dev)
+    st = L.ut_block_mask(ctypes.byref(shape), mode, _p(q), _p(k), float(rho), _p(bitmap), _p(row_ptr), _p(col_idx),
+                         col_cap, _p(col_ptr), _p(row_idx), _p(ws), ws.numel(), _p(status), _stream())
+    _check("ut_block_mask", st)
+    return row_ptr, col_idx, col_ptr, row_idx
+
+
+def ut_bsattn_fwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, row_ptr: torch.Tensor, col_idx: torch.Tensor,
+                  block: int, softmax_scale: Optional[float] = None, o: Optional[torch.Tensor] = None,
+                  lse: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None):
+    """Block-sparse attention forward.  Returns (O [N,H,d], LSE [H,N] fp32)."""
+    shape = attn_shape(q, block)
+    N, H, d = q.shape
+    scale = d ** -0.5 if softmax_scale is None else float(softmax_scale)
+    if o is None:
+        o = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty((H, N), dtype=torch.float32, device=q.device)
+    st = lib().ut_bsattn_fwd(ctypes.byref(shape), _p(q), _p(k), _p(v), _p(row_ptr), _p(col_idx), scale, _p(o),
+                             _p(lse), _p(status), _stream())
+    _check("ut_bsattn_fwd", st)
+    return o, lse
+
+
+def ut_bsattn_bwd(q, k, v, o, lse, dout, row_ptr, col_idx, col_ptr_t, row_idx_t, block: int,
+                  softmax_scale: Optional[float] = None, dq=None, dk=None, dv=None, ws=None, status=None):
+    """Gradient of ut_bsattn_fwd.  Returns (dQ, dK, dV)."""
+    shape = attn_shape(q, block)
+    d = q.shape[2]
+    scale = d ** -0.5 if softmax_scale is None else float(softmax_scale)
+    dq = torch.empty_like(q) if dq is None else dq
+    dk = torch.empty_like(k) if dk is None else dk
+    dv = torch.empty_like(v) if dv is None else dv
+    L = lib()
+    wsb = L.ut_bsattn_bwd_workspace_size(ctypes.byref(shape))
+    if ws is None:
+        ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device=q.device)
+    st = L.ut_bsattn_bwd(ctypes.byref(shape), _p(q), _p(k), _p(v), _p(o), _p(lse), _p(dout), _p(row_ptr),
+                         _p(col_idx), _p(col_ptr_t), _p(row_idx_t), scale, _p(dq), _p(dk), _p(dv), _p(ws),
+                         ws.numel(), _p(status), _stream())
+    _check("ut_bsattn_bwd", st)
+    return dq, dk, dv

@@ -1,0 +1,103 @@
+"""Host-side checks of the C ABI (no GPU needed): the library loads, exports
+every declared entry point, and rejects bad arguments before launching."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    import __graft_entry__ as g
+    g.build()
+    from paper_2609_23169_gb300 import ultratex
+    return ultratex.lib()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "ultratex.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(ut_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(L):
+    names = declared_functions()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(L, n), n
+    from paper_2609_23169_gb300 import ultratex
+    assert sorted(ultratex.EXPORTS) == sorted(names)
+
+
+def test_strerror_and_topk_count(L):
+    from paper_2609_23169_gb300 import ultratex as u
+    assert L.ut_strerror(u.UT_ERR_TIMEOUT) == b"device wait timed out"
+    import oracle.ultratex_oracle as o
+    for rho in (0.05, 0.1, 0.12, 0.2, 0.25, 0.3, 0.5, 0.7, 1.0):
+        for nk in (1, 3, 8, 10, 61, 188, 666, 1332):
+            assert u.ut_topk_count(rho, nk) == o.k_rho(rho, nk), (rho, nk)
+
+
+def _shape(u, N=256, H=2, d=64, b=32, dtype=1, rs=None):
+    return u.AttnShape(N, H, d, b, dtype, H * d if rs is None else rs)
+
+
+def test_argument_errors_are_caught_on_host(L):
+    from paper_2609_23169_gb300 import ultratex as u
+    bogus = ctypes.c_void_p(16 * 1024)   # never dereferenced: every call must fail validation first
+    S = ctypes.byref
+    # unsupported head dim / dtype / block
+    assert L.ut_bsattn_fwd(S(_shape(u, d=96)), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
+        == u.UT_ERR_UNSUPPORTED
+    assert L.ut_bsattn_fwd(S(_shape(u, dtype=7)), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
+        == u.UT_ERR_INVALID_ARG
+    assert L.ut_bsattn_fwd(S(_shape(u, dtype=0, b=64)), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None,
+                           None) == u.UT_ERR_UNSUPPORTED
+    # bad row stride, null pointers, bad scale, misalignment
+    assert L.ut_bsattn_fwd(S(_shape(u, rs=100)), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
+        == u.UT_ERR_INVALID_ARG
+    assert L.ut_bsattn_fwd(S(_shape(u)), None, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
+        == u.UT_ERR_INVALID_ARG
+    assert L.ut_bsattn_fwd(S(_shape(u)), bogus, bogus, bogus, bogus, bogus, -1.0, bogus, bogus, None, None) \
+        == u.UT_ERR_INVALID_ARG
+    odd = ctypes.c_void_p(16 * 1024 + 4)
+    assert L.ut_bsattn_fwd(S(_shape(u)), odd, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
+        == u.UT_ERR_INVALID_ARG
+    # N = 0 is a no-op
+    assert L.ut_bsattn_fwd(S(_shape(u, N=0)), None, None, None, None, None, 0.1, None, None, None, None) == u.UT_OK
+    # compaction: row bytes not a multiple of 16, too many tensors, no workspace
+    arr = (ctypes.c_void_p * 1)(bogus.value)
+    assert L.ut_fg_compact(bogus, 100, 1, arr, arr, 24, 100, bogus, bogus, bogus, 64, None, None) \
+        == u.UT_ERR_INVALID_ARG
+    assert L.ut_fg_compact(bogus, 100, 9, arr, arr, 32, 100, bogus, bogus, bogus, 64, None, None) \
+        == u.UT_ERR_INVALID_ARG
+    assert L.ut_fg_compact(bogus, 100, 1, arr, arr, 32, 100, bogus, bogus, None, 0, None, None) \
+        == u.UT_ERR_INVALID_ARG
+    # scatter: n > T, unknown mode, FILL without a row
+    assert L.ut_fg_scatter(bogus, 10, 1, arr, arr, 32, u.UT_BG_KEEP, None, 5, None) == u.UT_ERR_INVALID_ARG
+    assert L.ut_fg_scatter(bogus, 1, 1, arr, arr, 32, 9, None, 5, None) == u.UT_ERR_INVALID_ARG
+    assert L.ut_fg_scatter(bogus, 1, 1, arr, arr, 32, u.UT_BG_FILL, None, 5, None) == u.UT_ERR_INVALID_ARG
+    # block mask: rho out of range, capacity too small for Top-K, bitmap mode without a status word
+    sh = _shape(u, N=256, b=32)
+    wsb = L.ut_block_mask_workspace_size(S(sh), u.UT_MASK_TOPK)
+    assert wsb > 0
+    assert L.ut_block_mask(S(sh), u.UT_MASK_TOPK, bogus, bogus, 0.0, None, bogus, bogus, 100, None, None, bogus, wsb,
+                           None, None) == u.UT_ERR_INVALID_ARG
+    assert L.ut_block_mask(S(sh), u.UT_MASK_TOPK, bogus, bogus, 0.5, None, bogus, bogus, 3, None, None, bogus, wsb,
+                           None, None) == u.UT_ERR_CAPACITY
+    assert L.ut_block_mask(S(sh), u.UT_MASK_BITMAP, None, None, 0.0, bogus, bogus, bogus, 100, None, None, bogus,
+                           wsb, None, None) == u.UT_ERR_INVALID_ARG
+    # backward needs the transposed lists
+    assert L.ut_bsattn_bwd(S(_shape(u)), bogus, bogus, bogus, bogus, bogus, bogus, bogus, bogus, None, None, 0.1,
+                           bogus, bogus, bogus, bogus, 1 << 20, None, None) == u.UT_ERR_INVALID_ARG
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    from paper_2609_23169_gb300 import ultratex as u
+    monkeypatch.setattr(u, "_lib", None)
+    monkeypatch.setattr(u, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        u.lib()
