@@ -299,8 +299,8 @@ def run_ours(args, rank, world, local_rank):
 
 def hp_launches(hp) -> int:
     """Kernel launches of one HotPath.step (compaction 3, Top-K lists 3 + transpose 3,
-    forward 1, backward 4, scatter 2)."""
-    return 3 + 6 + 1 + 4 + 2
+    forward 1, backward 3 (preprocess, dK/dV, dQ), scatter 2)."""
+    return 3 + 6 + 1 + 3 + 2
 
 
 # ------------------------------------------------------------------- oracle

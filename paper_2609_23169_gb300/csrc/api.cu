@@ -207,14 +207,14 @@ size_t ut_bsattn_bwd_workspace_size(const ut_attn_shape* shape) {
   if (check_shape(shape, &nq) != UT_OK) return 0;
   AttnProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride,
                 nq, 1.f};
-  return attn_bwd_simt_ws(p) + 256;
+  const size_t a = attn_bwd_simt_ws(p), b = attn_bwd_tc_ws(p);
+  return (a > b ? a : b) + 256;
 }
 
 ut_status ut_bsattn_bwd(const ut_attn_shape* shape, const void* q, const void* k, const void* v, const void* o,
                         const float* lse, const void* dout, const int32_t* row_ptr, const int32_t* col_idx,
                         const int32_t* col_ptr_t, const int32_t* row_idx_t, float softmax_scale, void* dq, void* dk,
                         void* dv, void* ws, size_t ws_bytes, int32_t* dev_status, void* stream) {
-  (void)dev_status;
   int nq = 0;
   ut_status st = check_shape(shape, &nq);
   if (st != UT_OK) return st;
@@ -226,10 +226,18 @@ ut_status ut_bsattn_bwd(const ut_attn_shape* shape, const void* q, const void* k
     return UT_ERR_INVALID_ARG;
   AttnProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride,
                 nq, softmax_scale};
-  if (!ws || ws_bytes < attn_bwd_simt_ws(p)) return UT_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  return from_cuda(launch_attn_bwd_simt(p, q, k, v, o, lse, dout, row_ptr, col_idx, col_ptr_t, row_idx_t, dq, dk,
-                                        dv, ws, s));
+  if (shape->dtype == UT_F32) {
+    if (!ws || ws_bytes < attn_bwd_simt_ws(p)) return UT_ERR_INVALID_ARG;
+    return from_cuda(launch_attn_bwd_simt(p, q, k, v, o, lse, dout, row_ptr, col_idx, col_ptr_t, row_idx_t, dq, dk,
+                                          dv, ws, s));
+  }
+  if (!ws || ws_bytes < attn_bwd_tc_ws(p) || !aligned16(ws)) return UT_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(dout) || !aligned16(dq) ||
+      !aligned16(dk) || !aligned16(dv))
+    return UT_ERR_INVALID_ARG;
+  return from_cuda(launch_attn_bwd_tc(p, q, k, v, o, lse, dout, row_ptr, col_idx, col_ptr_t, row_idx_t, dq, dk, dv,
+                                      ws, dev_status, wait_timeout_ns(), device_sms(), s));
 }
 
 }  // extern "C"

@@ -1,0 +1,723 @@
+// Block-sparse attention backward on the tcgen05 tensor cores.
+//
+// With P = exp(S - LSE) recomputed from the forward's row normalisers and
+// D_r = dO_r . O_r:
+//   dV = P^T dO,   dS = P o (dO V^T - D),   dQ = scale * dS K,   dK = scale * dS^T Q
+// over the retained block pairs only.  Two persistent kernels, no atomics:
+//
+//   bwd_pre_kernel    D_r and LSE_r * log2(e) per (head, row) into a padded
+//                     [H, N_q*128] workspace (padding rows: D = 0, LSE = +inf
+//                     so that they contribute P = 0).
+//   bwd_dq_kernel     item (h, query block i) over its key list S_i:
+//                       S = Q K_j^T, dP = dO V_j^T   (TMEM)
+//                       dS -> bf16, 128B-swizzled shared tile
+//                       dQ += dS K_j                 (TMEM accumulator)
+//   bwd_dkdv_kernel   item (h, key block j) over the transposed list (query
+//                     blocks i with j in S_i):
+//                       S^T = K_j Q_i^T, dP^T = V_j dO_i^T   (TMEM)
+//                       P^T, then dS^T -> bf16 shared tile (one buffer, reused)
+//                       dV += P^T dO_i, dK += dS^T Q_i       (TMEM accumulators)
+//
+// Roles as in the forward: warp 0 TMA producer, warp 1 TMEM owner + MMA
+// issuer, warps 2-5 elementwise (thread = TMEM lane = one row of the tile).
+// All waits are bounded (UT_ERR_TIMEOUT on expiry, then drain and return).
+#include "common.cuh"
+#include "kernels.h"
+
+namespace ut {
+
+constexpr int kTile = 128;
+constexpr int kBwdThreads = 192;
+constexpr uint32_t kChunk = 128 * 128;  // one 128-row x 128-byte swizzled sub-tile
+
+// ------------------------------------------------------------- preprocess
+// One warp per (padded) row r; a half-warp per head (8 bf16 per lane).
+__global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __restrict__ o,
+                                                      const __nv_bfloat16* __restrict__ dout,
+                                                      const float* __restrict__ lse, int64_t N, int64_t Np, int H,
+                                                      int d, int64_t rs, float* __restrict__ lse2,
+                                                      float* __restrict__ dsum) {
+  const int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (r >= Np) return;
+  const int lane = threadIdx.x & 31;
+  const int lanes_per_head = d / 8;           // 16 (d=128) or 8 (d=64)
+  const int heads_per_iter = 32 / lanes_per_head;
+  for (int h0 = 0; h0 < H; h0 += heads_per_iter) {
+    const int h = h0 + lane / lanes_per_head;
+    float s = 0.f;
+    if (r < N && h < H) {
+      const int64_t off = r * rs + (int64_t)h * d + (lane % lanes_per_head) * 8;
+      uint4 a = *reinterpret_cast<const uint4*>(o + off);
+      uint4 b = *reinterpret_cast<const uint4*>(dout + off);
+      const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
+      const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        float2 x = __bfloat1622float2(pa[e]);
+        float2 y = __bfloat1622float2(pb[e]);
+        s = fmaf(x.x, y.x, s);
+        s = fmaf(x.y, y.y, s);
+      }
+    }
+    for (int off = lanes_per_head / 2; off; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if ((lane % lanes_per_head) == 0 && h < H) {
+      dsum[(int64_t)h * Np + r] = r < N ? s : 0.f;
+      lse2[(int64_t)h * Np + r] = r < N ? lse[(int64_t)h * N + r] * 1.4426950408889634f : INFINITY;
+    }
+  }
+}
+
+struct BwdParams {
+  const int32_t* ptr;   // CSR row_ptr (dq) or CSC col_ptr (dkdv)
+  const int32_t* idx;   // col_idx (dq) or row_idx (dkdv)
+  const float* lse2;    // [H, Np]  LSE * log2(e)
+  const float* dsum;    // [H, Np]  D
+  __nv_bfloat16* out0;  // dq  | dv
+  __nv_bfloat16* out1;  //     | dk
+  int32_t* status;
+  int64_t N, Np, rs;
+  int H, nq, n_items;
+  float scale, scale_log2;
+  uint64_t timeout_ns;
+};
+
+// =========================================================================
+//                                  dQ
+// =========================================================================
+template <int D>
+struct DqSmem {
+  static constexpr int kC = D / 64;
+  static constexpr uint32_t kTileBytes = kTile * D * 2;
+  alignas(1024) uint8_t q[kTileBytes];
+  alignas(1024) uint8_t dout[kTileBytes];
+  alignas(1024) uint8_t k[2][kTileBytes];
+  alignas(1024) uint8_t v[2][kTileBytes];
+  alignas(1024) uint8_t ds[kTile * kTile * 2];
+  uint64_t qd_full, qd_empty;
+  uint64_t k_full[2], v_full[2], kv_empty[2];
+  uint64_t sp_full, sp_empty, ds_full, dq_mma_done, dq_empty, mma_done;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kBwdThreads, 1)
+    bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                  const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+                  const BwdParams prm) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  DqSmem<D>& sm = *reinterpret_cast<DqSmem<D>*>(smem_raw);
+  constexpr int C = DqSmem<D>::kC;
+  constexpr uint32_t TB = DqSmem<D>::kTileBytes;
+  const uint32_t warp = warp_id(), lane = lane_id();
+  volatile int* abort_flag = &sm.abort_flag;
+  if ((smem_u32(smem_raw) & 1023u) != 0) {  // the swizzled tiles need 1024-byte alignment
+    if (threadIdx.x == 0) set_status(prm.status, UT_ERR_INVALID_ARG);
+    return;
+  }
+  if (threadIdx.x == 0) {
+    mbar_init(&sm.qd_full, 1);
+    mbar_init(&sm.qd_empty, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.k_full[s], 1);
+      mbar_init(&sm.v_full[s], 1);
+      mbar_init(&sm.kv_empty[s], 1);
+    }
+    mbar_init(&sm.sp_full, 1);
+    mbar_init(&sm.sp_empty, 4);
+    mbar_init(&sm.ds_full, 4);
+    mbar_init(&sm.dq_mma_done, 1);
+    mbar_init(&sm.dq_empty, 4);
+    mbar_init(&sm.mma_done, 1);
+    sm.abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  const int G = gridDim.x;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      tma_prefetch_desc(&tm_do);
+      const uint64_t pol_kv = policy_evict_last(), pol_q = policy_evict_first();
+      uint32_t qi = 0, kv = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+        const int h = w / prm.nq, i = w % prm.nq;
+        const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+        if (L <= 0) continue;
+        if (!(ok = mbar_wait(&sm.qd_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        mbar_expect_tx(&sm.qd_full, 2 * TB);
+        for (int c = 0; c < C; ++c) {
+          tma_load_2d(sm.q + c * kChunk, &tm_q, &sm.qd_full, h * D + c * 64, i * kTile, pol_q);
+          tma_load_2d(sm.dout + c * kChunk, &tm_do, &sm.qd_full, h * D + c * 64, i * kTile, pol_q);
+        }
+        ++qi;
+        for (int t = 0; t < L; ++t, ++kv) {
+          const int j = prm.idx[beg + t];
+          const int st = kv & 1;
+          const uint32_t n = kv >> 1;
+          if (!(ok = mbar_wait(&sm.kv_empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&sm.k_full[st], TB);
+          for (int c = 0; c < C; ++c)
+            tma_load_2d(sm.k[st] + c * kChunk, &tm_k, &sm.k_full[st], h * D + c * 64, j * kTile, pol_kv);
+          mbar_expect_tx(&sm.v_full[st], TB);
+          for (int c = 0; c < C; ++c)
+            tma_load_2d(sm.v[st] + c * kChunk, &tm_v, &sm.v_full[st], h * D + c * 64, j * kTile, pol_kv);
+        }
+      }
+      const uint64_t t0 = globaltimer();
+      auto drain = [&](uint64_t* bar, uint32_t parity) {
+        while (!mbar_try_wait(bar, parity))
+          if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+      };
+      if (qi > 0) drain(&sm.qd_full, (qi - 1) & 1);
+      for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) {
+        drain(&sm.k_full[u & 1], (u >> 1) & 1);
+        drain(&sm.v_full[u & 1], (u >> 1) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
+      constexpr uint32_t idesc_dq = idesc_bf16_f32(kTile, D, false, true);
+      const uint32_t q_addr = smem_u32(sm.q), do_addr = smem_u32(sm.dout), ds_addr = smem_u32(sm.ds);
+      uint32_t qi = 0, kv0 = 0, sc0 = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+        const int L = prm.ptr[w + 1] - prm.ptr[w];
+        if (L <= 0) continue;
+        if (!(ok = mbar_wait(&sm.qd_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        for (int t = 0; t <= L && ok; ++t) {
+          if (t < L) {
+            const uint32_t kv = kv0 + t, st = kv & 1, n = kv >> 1;
+            const uint32_t sc = sc0 + t;
+            if (!(ok = mbar_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.sp_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+            const uint32_t k_addr = smem_u32(sm.k[st]), v_addr = smem_u32(sm.v[st]);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss(tmem, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024), idesc_s,
+                          kk > 0);
+            }
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss(tmem + 128, sdesc_sw128(do_addr + off, 16, 1024), sdesc_sw128(v_addr + off, 16, 1024),
+                          idesc_s, kk > 0);
+            }
+            mma_commit(&sm.sp_full);
+            if (t == L - 1) mma_commit(&sm.qd_empty);
+          }
+          if (t >= 1) {
+            const uint32_t u = t - 1;
+            const uint32_t kv = kv0 + u, st = kv & 1;
+            const uint32_t sc = sc0 + u;
+            if (!(ok = mbar_wait(&sm.ds_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (u == 0 && !(ok = mbar_wait(&sm.dq_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+              break;
+            tc_fence_after();
+            const uint32_t k_addr = smem_u32(sm.k[st]);
+#pragma unroll
+            for (int kk = 0; kk < kTile / 16; ++kk) {
+              const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss(tmem + 256, sdesc_sw128(ds_addr + aoff, 16, 1024),
+                          sdesc_sw128(k_addr + kk * 2048, kChunk, 1024), idesc_dq, (u > 0 || kk > 0));
+            }
+            mma_commit(&sm.dq_mma_done);
+            mma_commit(&sm.kv_empty[st]);
+          }
+        }
+        kv0 += L;
+        sc0 += L;
+        ++qi;
+      }
+      mma_commit(&sm.mma_done);
+      const uint64_t t0 = globaltimer();
+      while (!mbar_try_wait(&sm.mma_done, 0))
+        if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+    }
+  } else {
+    const uint32_t quarter = warp & 3;
+    const uint32_t row = quarter * 32 + lane;
+    const uint32_t lane_base = (quarter * 32) << 16;
+    const float c = prm.scale_log2;
+    uint32_t sc0 = 0;
+    bool ok = true;
+    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+      const int h = w / prm.nq, i = w % prm.nq;
+      const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+      const int64_t grow = (int64_t)i * kTile + row;
+      const bool row_ok = grow < prm.N;
+      __nv_bfloat16* orow = prm.out0 + grow * prm.rs + (int64_t)h * D;
+      if (L <= 0) {
+        if (row_ok)
+          for (int e = 0; e < D; e += 8) *reinterpret_cast<uint4*>(orow + e) = make_uint4(0, 0, 0, 0);
+        continue;
+      }
+      const float lse2 = prm.lse2[(int64_t)h * prm.Np + grow];
+      const float Dr = prm.dsum[(int64_t)h * prm.Np + grow];
+      for (int t = 0; t < L; ++t) {
+        const uint32_t sc = sc0 + t;
+        if (!(ok = warp_wait(&sm.sp_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
+        const int j = prm.idx[beg + t];
+        const int64_t nv = prm.N - (int64_t)j * kTile;
+        float p[kTile];
+#pragma unroll
+        for (int g = 0; g < kTile / 32; ++g) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + g * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int x = 0; x < 32; ++x) {
+            const int col = g * 32 + x;
+            p[col] = col < nv ? ex2_approx(fmaf(__uint_as_float(r[x]), c, -lse2)) : 0.f;
+          }
+        }
+        // dS buffer is free once the previous tile's dQ MMA finished
+        if (!(ok = warp_wait(&sm.dq_mma_done, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        const uint32_t ds_row = smem_u32(sm.ds) + row * 128;
+#pragma unroll
+        for (int g = 0; g < kTile / 32; ++g) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + 128 + g * 32, r);
+          tmem_wait_ld();
+          uint32_t pk[16];
+#pragma unroll
+          for (int x = 0; x < 32; x += 2) {
+            const float d0 = p[g * 32 + x] * (__uint_as_float(r[x]) - Dr);
+            const float d1 = p[g * 32 + x + 1] * (__uint_as_float(r[x + 1]) - Dr);
+            pk[x / 2] = pack_bf16x2(d0, d1);
+          }
+#pragma unroll
+          for (int u4 = 0; u4 < 4; ++u4) {
+            const uint32_t u = g * 4 + u4;  // 16-byte unit (8 keys) within the 128-key row
+            const uint32_t chunk = u >> 3, unit = u & 7;
+            st_shared_v4(ds_row + chunk * kChunk + ((unit ^ (row & 7)) << 4), pk[4 * u4], pk[4 * u4 + 1],
+                         pk[4 * u4 + 2], pk[4 * u4 + 3]);
+          }
+        }
+        tc_fence_before();
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&sm.sp_empty);
+          mbar_arrive(&sm.ds_full);
+        }
+      }
+      if (!ok) break;
+      const uint32_t last = sc0 + L - 1;
+      if (!(ok = warp_wait(&sm.dq_mma_done, last & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+      tc_fence_after();
+#pragma unroll
+      for (int g = 0; g < D / 32; ++g) {
+        uint32_t r[32];
+        tmem_ld32(tmem + lane_base + 256 + g * 32, r);
+        tmem_wait_ld();
+        if (row_ok) {
+#pragma unroll
+          for (int x = 0; x < 32; x += 8) {
+            uint4 v;
+            v.x = pack_bf16x2(__uint_as_float(r[x + 0]) * prm.scale, __uint_as_float(r[x + 1]) * prm.scale);
+            v.y = pack_bf16x2(__uint_as_float(r[x + 2]) * prm.scale, __uint_as_float(r[x + 3]) * prm.scale);
+            v.z = pack_bf16x2(__uint_as_float(r[x + 4]) * prm.scale, __uint_as_float(r[x + 5]) * prm.scale);
+            v.w = pack_bf16x2(__uint_as_float(r[x + 6]) * prm.scale, __uint_as_float(r[x + 7]) * prm.scale);
+            *reinterpret_cast<uint4*>(orow + g * 32 + x) = v;
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.dq_empty);
+      sc0 += L;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// =========================================================================
+//                                dK, dV
+// =========================================================================
+template <int D>
+struct DkdvSmem {
+  static constexpr int kC = D / 64;
+  static constexpr uint32_t kTileBytes = kTile * D * 2;
+  alignas(1024) uint8_t k[kTileBytes];
+  alignas(1024) uint8_t v[kTileBytes];
+  alignas(1024) uint8_t q[2][kTileBytes];
+  alignas(1024) uint8_t dout[2][kTileBytes];
+  alignas(1024) uint8_t pds[kTile * kTile * 2];   // P^T, then dS^T, of the current pair
+  float lse2[2][kTile];
+  float dsum[2][kTile];
+  uint64_t kv_full, kv_empty;
+  uint64_t qd_full[2], qd_empty[2];
+  uint64_t sp_full, sp_empty, pt_full, pt_done, dst_full, ds_done, acc_full, acc_empty, mma_done;
+  uint64_t rowvec_full[2];   // the 128 elementwise threads staged this pair's LSE / D
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kBwdThreads, 1)
+    bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+                    const BwdParams prm) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  DkdvSmem<D>& sm = *reinterpret_cast<DkdvSmem<D>*>(smem_raw);
+  constexpr int C = DkdvSmem<D>::kC;
+  constexpr uint32_t TB = DkdvSmem<D>::kTileBytes;
+  const uint32_t warp = warp_id(), lane = lane_id();
+  volatile int* abort_flag = &sm.abort_flag;
+  if ((smem_u32(smem_raw) & 1023u) != 0) {
+    if (threadIdx.x == 0) set_status(prm.status, UT_ERR_INVALID_ARG);
+    return;
+  }
+  if (threadIdx.x == 0) {
+    mbar_init(&sm.kv_full, 1);
+    mbar_init(&sm.kv_empty, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.qd_full[s], 1);
+      mbar_init(&sm.qd_empty[s], 1);
+    }
+    mbar_init(&sm.sp_full, 1);
+    mbar_init(&sm.sp_empty, 4);
+    mbar_init(&sm.pt_full, 4);
+    mbar_init(&sm.pt_done, 1);
+    mbar_init(&sm.dst_full, 4);
+    mbar_init(&sm.ds_done, 1);
+    mbar_init(&sm.acc_full, 1);
+    mbar_init(&sm.acc_empty, 4);
+    mbar_init(&sm.mma_done, 1);
+    mbar_init(&sm.rowvec_full[0], 128);
+    mbar_init(&sm.rowvec_full[1], 128);
+    sm.abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  const int G = gridDim.x;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      tma_prefetch_desc(&tm_do);
+      const uint64_t pol_qd = policy_evict_last(), pol_kv = policy_evict_first();
+      uint32_t ki = 0, qd = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+        const int h = w / prm.nq, j = w % prm.nq;
+        const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+        if (L <= 0) continue;
+        if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        mbar_expect_tx(&sm.kv_full, 2 * TB);
+        for (int c = 0; c < C; ++c) {
+          tma_load_2d(sm.k + c * kChunk, &tm_k, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
+          tma_load_2d(sm.v + c * kChunk, &tm_v, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
+        }
+        ++ki;
+        for (int t = 0; t < L; ++t, ++qd) {
+          const int i = prm.idx[beg + t];
+          const int st = qd & 1;
+          const uint32_t n = qd >> 1;
+          if (!(ok = mbar_wait(&sm.qd_empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&sm.qd_full[st], 2 * TB);
+          for (int c = 0; c < C; ++c) {
+            tma_load_2d(sm.q[st] + c * kChunk, &tm_q, &sm.qd_full[st], h * D + c * 64, i * kTile, pol_qd);
+            tma_load_2d(sm.dout[st] + c * kChunk, &tm_do, &sm.qd_full[st], h * D + c * 64, i * kTile, pol_qd);
+          }
+        }
+      }
+      const uint64_t t0 = globaltimer();
+      auto drain = [&](uint64_t* bar, uint32_t parity) {
+        while (!mbar_try_wait(bar, parity))
+          if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+      };
+      if (ki > 0) drain(&sm.kv_full, (ki - 1) & 1);
+      for (uint32_t u = (qd >= 2 ? qd - 2 : 0); u < qd; ++u) drain(&sm.qd_full[u & 1], (u >> 1) & 1);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
+      constexpr uint32_t idesc_acc = idesc_bf16_f32(kTile, D, false, true);
+      const uint32_t k_addr = smem_u32(sm.k), v_addr = smem_u32(sm.v), pds_addr = smem_u32(sm.pds);
+      uint32_t ki = 0, qd0 = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+        const int L = prm.ptr[w + 1] - prm.ptr[w];
+        if (L <= 0) continue;
+        if (!(ok = mbar_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        for (int t = 0; t <= L && ok; ++t) {
+          if (t < L) {
+            const uint32_t qd = qd0 + t, st = qd & 1, n = qd >> 1;
+            if (!(ok = mbar_wait(&sm.qd_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.sp_empty, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+            const uint32_t q_addr = smem_u32(sm.q[st]), do_addr = smem_u32(sm.dout[st]);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss(tmem, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024), idesc_s,
+                          kk > 0);
+            }
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss(tmem + 128, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
+                          idesc_s, kk > 0);
+            }
+            mma_commit(&sm.sp_full);
+            if (t == L - 1) mma_commit(&sm.kv_empty);
+          }
+          if (t >= 1) {
+            const uint32_t u = t - 1;
+            const uint32_t qd = qd0 + u, st = qd & 1;
+            const uint32_t q_addr = smem_u32(sm.q[st]), do_addr = smem_u32(sm.dout[st]);
+            if (!(ok = mbar_wait(&sm.pt_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (u == 0 && !(ok = mbar_wait(&sm.acc_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+              break;
+            tc_fence_after();
+#pragma unroll
+            for (int kk = 0; kk < kTile / 16; ++kk) {
+              const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss(tmem + 256, sdesc_sw128(pds_addr + aoff, 16, 1024),
+                          sdesc_sw128(do_addr + kk * 2048, kChunk, 1024), idesc_acc, (u > 0 || kk > 0));
+            }
+            mma_commit(&sm.pt_done);
+            if (!(ok = mbar_wait(&sm.dst_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+#pragma unroll
+            for (int kk = 0; kk < kTile / 16; ++kk) {
+              const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss(tmem + 384, sdesc_sw128(pds_addr + aoff, 16, 1024),
+                          sdesc_sw128(q_addr + kk * 2048, kChunk, 1024), idesc_acc, (u > 0 || kk > 0));
+            }
+            mma_commit(&sm.ds_done);
+            mma_commit(&sm.qd_empty[st]);
+          }
+        }
+        mma_commit(&sm.acc_full);
+        qd0 += L;
+        ++ki;
+      }
+      mma_commit(&sm.mma_done);
+      const uint64_t t0 = globaltimer();
+      while (!mbar_try_wait(&sm.mma_done, 0))
+        if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+    }
+  } else {
+    const uint32_t quarter = warp & 3;
+    const uint32_t krow = quarter * 32 + lane;          // key row of the tile = TMEM lane
+    const uint32_t tid = threadIdx.x - 64;               // 0..127 within the elementwise group
+    const uint32_t lane_base = (quarter * 32) << 16;
+    const float c = prm.scale_log2;
+    uint32_t qd0 = 0, ki = 0;
+    bool ok = true;
+    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+      const int h = w / prm.nq, j = w % prm.nq;
+      const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+      const int64_t gk = (int64_t)j * kTile + krow;
+      const bool row_ok = gk < prm.N;
+      __nv_bfloat16* dv_row = prm.out0 + gk * prm.rs + (int64_t)h * D;
+      __nv_bfloat16* dk_row = prm.out1 + gk * prm.rs + (int64_t)h * D;
+      if (L <= 0) {
+        if (row_ok)
+          for (int e = 0; e < D; e += 8) {
+            *reinterpret_cast<uint4*>(dv_row + e) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(dk_row + e) = make_uint4(0, 0, 0, 0);
+          }
+        continue;
+      }
+      for (int t = 0; t < L; ++t) {
+        const uint32_t qd = qd0 + t;
+        const int i = prm.idx[beg + t];
+        // this pair's query-row LSE*log2e and D into the shared double buffer
+        // (buffer qd&1 was last read in pair qd-2, which every thread finished
+        //  before arriving for pair qd-1)
+        sm.lse2[qd & 1][tid] = prm.lse2[(int64_t)h * prm.Np + (int64_t)i * kTile + tid];
+        sm.dsum[qd & 1][tid] = prm.dsum[(int64_t)h * prm.Np + (int64_t)i * kTile + tid];
+        mbar_arrive(&sm.rowvec_full[qd & 1]);
+        if (!(ok = warp_wait(&sm.rowvec_full[qd & 1], (qd >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
+          break;
+        const float* ls = sm.lse2[qd & 1];
+        const float* ds_v = sm.dsum[qd & 1];
+        if (!(ok = warp_wait(&sm.sp_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
+        float p[kTile];
+#pragma unroll
+        for (int g = 0; g < kTile / 32; ++g) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + g * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int x = 0; x < 32; ++x) p[g * 32 + x] = ex2_approx(fmaf(__uint_as_float(r[x]), c, -ls[g * 32 + x]));
+        }
+        // the shared P/dS tile is free once the previous pair's dK MMA finished
+        if (!(ok = warp_wait(&sm.ds_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        const uint32_t pds_row = smem_u32(sm.pds) + krow * 128;
+#pragma unroll
+        for (int u = 0; u < kTile / 8; ++u) {
+          const uint32_t chunk = u >> 3, unit = u & 7;
+          st_shared_v4(pds_row + chunk * kChunk + ((unit ^ (krow & 7)) << 4), pack_bf16x2(p[8 * u], p[8 * u + 1]),
+                       pack_bf16x2(p[8 * u + 2], p[8 * u + 3]), pack_bf16x2(p[8 * u + 4], p[8 * u + 5]),
+                       pack_bf16x2(p[8 * u + 6], p[8 * u + 7]));
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.pt_full);
+        uint32_t dsk[kTile / 2];
+#pragma unroll
+        for (int g = 0; g < kTile / 32; ++g) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + 128 + g * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int x = 0; x < 32; x += 2) {
+            const int col = g * 32 + x;
+            dsk[col / 2] = pack_bf16x2(p[col] * (__uint_as_float(r[x]) - ds_v[col]),
+                                       p[col + 1] * (__uint_as_float(r[x + 1]) - ds_v[col + 1]));
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.sp_empty);
+        // overwrite P^T with dS^T once the dV MMA has read P^T
+        if (!(ok = warp_wait(&sm.pt_done, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+#pragma unroll
+        for (int u = 0; u < kTile / 8; ++u) {
+          const uint32_t chunk = u >> 3, unit = u & 7;
+          st_shared_v4(pds_row + chunk * kChunk + ((unit ^ (krow & 7)) << 4), dsk[4 * u], dsk[4 * u + 1],
+                       dsk[4 * u + 2], dsk[4 * u + 3]);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.dst_full);
+      }
+      if (!ok) break;
+      if (!(ok = warp_wait(&sm.acc_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+      tc_fence_after();
+#pragma unroll
+      for (int part = 0; part < 2; ++part) {
+        __nv_bfloat16* dst = part == 0 ? dv_row : dk_row;
+        const float f = part == 0 ? 1.0f : prm.scale;
+#pragma unroll
+        for (int g = 0; g < D / 32; ++g) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + 256 + part * 128 + g * 32, r);
+          tmem_wait_ld();
+          if (row_ok) {
+#pragma unroll
+            for (int x = 0; x < 32; x += 8) {
+              uint4 v;
+              v.x = pack_bf16x2(__uint_as_float(r[x + 0]) * f, __uint_as_float(r[x + 1]) * f);
+              v.y = pack_bf16x2(__uint_as_float(r[x + 2]) * f, __uint_as_float(r[x + 3]) * f);
+              v.z = pack_bf16x2(__uint_as_float(r[x + 4]) * f, __uint_as_float(r[x + 5]) * f);
+              v.w = pack_bf16x2(__uint_as_float(r[x + 6]) * f, __uint_as_float(r[x + 7]) * f);
+              *reinterpret_cast<uint4*>(dst + g * 32 + x) = v;
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.acc_empty);
+      qd0 += L;
+      ++ki;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// ----------------------------------------------------------------- launcher
+size_t attn_bwd_tc_ws(const AttnProblem& p) {
+  const size_t Np = (size_t)p.nq * kTile;
+  return 2 * (size_t)p.H * Np * sizeof(float);
+}
+
+template <int D>
+static cudaError_t launch_bwd_d(const AttnProblem& p, const CUtensorMap* tm, BwdParams prm_dq, BwdParams prm_kv,
+                                int sms, cudaStream_t s) {
+  const int n_items = p.H * p.nq;
+  const int grid = n_items < sms ? n_items : sms;
+  const size_t smem_dq = sizeof(DqSmem<D>);
+  const size_t smem_kv = sizeof(DkdvSmem<D>);
+  cudaError_t e = cudaFuncSetAttribute(bwd_dq_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_dq);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(bwd_dkdv_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_kv);
+  if (e != cudaSuccess) return e;
+  bwd_dkdv_kernel<D><<<grid, kBwdThreads, smem_kv, s>>>(tm[0], tm[1], tm[2], tm[3], prm_kv);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  bwd_dq_kernel<D><<<grid, kBwdThreads, smem_dq, s>>>(tm[0], tm[1], tm[2], tm[3], prm_dq);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* k, const void* v, const void* o,
+                               const float* lse, const void* dout, const int32_t* row_ptr, const int32_t* col_idx,
+                               const int32_t* col_ptr_t, const int32_t* row_idx_t, void* dq, void* dk, void* dv,
+                               void* ws, int32_t* status, uint64_t timeout_ns, int sms, cudaStream_t stream) {
+  if (p.nq == 0) return cudaSuccess;
+  const int64_t Np = (int64_t)p.nq * kTile;
+  float* lse2 = static_cast<float*>(ws);
+  float* dsum = lse2 + (size_t)p.H * Np;
+  bwd_pre_kernel<<<(unsigned)((Np + 7) / 8), 256, 0, stream>>>(
+      static_cast<const __nv_bfloat16*>(o), static_cast<const __nv_bfloat16*>(dout), lse, p.N, Np, p.H, p.d,
+      p.row_stride, lse2, dsum);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  CUtensorMap tm[4];
+  const uint64_t inner = (uint64_t)p.H * p.d, stride = (uint64_t)p.row_stride * 2;
+  const void* bases[4] = {q, k, v, dout};
+  for (int x = 0; x < 4; ++x)
+    if (!encode_tmap_2d_bf16(&tm[x], bases[x], inner, p.N, stride, 64, kTile)) return cudaErrorInvalidValue;
+  BwdParams a{};
+  a.lse2 = lse2;
+  a.dsum = dsum;
+  a.status = status;
+  a.N = p.N;
+  a.Np = Np;
+  a.rs = p.row_stride;
+  a.H = p.H;
+  a.nq = p.nq;
+  a.n_items = p.H * p.nq;
+  a.scale = p.scale;
+  a.scale_log2 = p.scale * 1.4426950408889634f;
+  a.timeout_ns = timeout_ns;
+  BwdParams pq = a, pk = a;
+  pq.ptr = row_ptr;
+  pq.idx = col_idx;
+  pq.out0 = static_cast<__nv_bfloat16*>(dq);
+  pk.ptr = col_ptr_t;
+  pk.idx = row_idx_t;
+  pk.out0 = static_cast<__nv_bfloat16*>(dv);
+  pk.out1 = static_cast<__nv_bfloat16*>(dk);
+  return p.d == 64 ? launch_bwd_d<64>(p, tm, pq, pk, sms, stream) : launch_bwd_d<128>(p, tm, pq, pk, sms, stream);
+}
+
+}  // namespace ut

@@ -55,6 +55,13 @@ cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* 
                                const int32_t* row_ptr, const int32_t* col_idx, void* o, float* lse, int32_t* status,
                                uint64_t timeout_ns, int sms, cudaStream_t stream);
 
+// attn_bwd_tc.cu (bf16 tcgen05 backward: preprocess, dK/dV, dQ)
+size_t attn_bwd_tc_ws(const AttnProblem& p);
+cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* k, const void* v, const void* o,
+                               const float* lse, const void* dout, const int32_t* row_ptr, const int32_t* col_idx,
+                               const int32_t* col_ptr_t, const int32_t* row_idx_t, void* dq, void* dk, void* dv,
+                               void* ws, int32_t* status, uint64_t timeout_ns, int sms, cudaStream_t stream);
+
 // tensor maps (api.cu)
 bool encode_tmap_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner_elems, uint64_t rows,
                          uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_rows);

@@ -207,3 +207,49 @@ def test_bwd_c512_four_heads_full():
     rq, rk, rv = o.bsattn_bwd(*(x.double().numpy() for x in (q, k, v, do)), rp, ci, w.block)
     for name, g, r in (("dQ", dq, rq), ("dK", dk, rk), ("dV", dv, rv)):
         print(name, assert_bf16_close(to_np(g), r, name))
+
+
+def _sampled_bwd_check(w, mode, key_heads=(0, 7)):
+    """Full-size forward + backward through the bench's path; sampled dQ rows in
+    every head and sampled dK/dV rows in two heads against the oracle."""
+    from paper_2609_23169_gb300 import path as P
+    mask = w.canvas_mask()
+    q, k, v, do = w.q(), w.k(), w.v(), w.dout()
+    bm = w.block_bitmap() if mode == "bitmap" else None
+    out = P.run_path(w, mask, q, k, v, do, bitmap=bm)
+    idx = np.flatnonzero(mask)
+    t = torch.from_numpy(idx)
+    qc, kc, vc, dc = (x[t].float().numpy() for x in (q, k, v, do))
+    nq = -(-w.N // w.block)
+    rp = out["row_ptr"][:w.heads * nq + 1].cpu().numpy()
+    ci = out["col_idx"][:int(rp[-1])].cpu().numpy()
+    rows = w.row_subsample(w.N, 0.005)
+    dq = out["dqc"].float().cpu().numpy()
+    dk = out["dkc"].float().cpu().numpy()
+    dv = out["dvc"].float().cpu().numpy()
+    got, ref = [], []
+    for h in range(w.heads):
+        got.append(dq[rows, h])
+        ref.append(o.bsattn_bwd_dq_rows(qc, kc, vc, dc, rp, ci, w.block, h, rows))
+    sq = assert_bf16_close(np.concatenate(got), np.concatenate(ref), "dQ " + w.name)
+    krows = rows[:24]
+    gk, gv, rk, rv = [], [], [], []
+    for h in key_heads:
+        a, b = o.bsattn_bwd_dkdv_rows(qc, kc, vc, dc, rp, ci, w.block, h, krows)
+        gk.append(dk[krows, h]); gv.append(dv[krows, h]); rk.append(a); rv.append(b)
+    sk = assert_bf16_close(np.concatenate(gk), np.concatenate(rk), "dK " + w.name)
+    sv = assert_bf16_close(np.concatenate(gv), np.concatenate(rv), "dV " + w.name)
+    # scatter (ZERO mode) put gradients at canvas positions and zeros elsewhere
+    gq = out["dq_canvas"]
+    assert torch.equal(gq[torch.from_numpy(idx[rows]).cuda()].float().cpu(), torch.from_numpy(dq[rows]))
+    bg = torch.from_numpy(np.flatnonzero(mask == 0)[:1000]).cuda()
+    assert torch.all(gq[bg] == 0)
+    return sq, sk, sv
+
+
+def test_bwd_c1024_sampled():
+    print(_sampled_bwd_check(CONFIGS["c1024"], "bitmap"))
+
+
+def test_bwd_c2048_sampled():
+    print(_sampled_bwd_check(CONFIGS["c2048"], "topk"))
