@@ -49,6 +49,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="c2048")
+    ap.add_argument("--heads", type=int, default=0, help="override the head count (small profiling cases)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -144,6 +145,8 @@ def run_ours(args, rank, world, local_rank):
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     w = CONFIGS[args.workload]
+    if args.heads:
+        w = w.with_(heads=args.heads)
     assert w.mask_mode == "topk", "the benchmark workload uses the Top-K rule"
     mask_np, q, k, v, do = make_inputs(w, dev)
     mask = torch.from_numpy(mask_np).to(dev)

@@ -96,6 +96,27 @@ def _ptr_array(ts: Sequence[torch.Tensor]):
     return (ctypes.c_void_p * len(ts))(*[t.data_ptr() for t in ts])
 
 
+def _row_bytes(ts: Sequence[torch.Tensor], min_rows: int, what: str) -> int:
+    """Common row size of a list of row-major tensors with at least min_rows rows.
+
+    The C entry points take one row size for the whole list, so every tensor
+    must share it; a mismatch would make the kernels read or write past a
+    smaller tensor."""
+    if len(ts) == 0:
+        raise ValueError(f"{what} is empty")
+    sizes = set()
+    for t in ts:
+        if not t.is_contiguous():
+            raise ValueError(f"{what}: tensors must be contiguous")
+        if t.shape[0] < min_rows:
+            raise ValueError(f"{what}: a tensor has {t.shape[0]} rows, fewer than {min_rows}")
+        sizes.add((t.numel() // max(1, t.shape[0])) * t.element_size() if t.shape[0] else -1)
+    sizes.discard(-1)
+    if len(sizes) > 1:
+        raise ValueError(f"{what}: tensors differ in row size {sorted(sizes)}; one call per row size")
+    return sizes.pop() if sizes else 16
+
+
 def _dtype_code(t: torch.Tensor) -> int:
     if t.dtype == torch.bfloat16:
         return UT_BF16
@@ -132,11 +153,15 @@ def ut_fg_compact(mask: torch.Tensor, srcs: Sequence[torch.Tensor], capacity: Op
                   status: Optional[torch.Tensor] = None):
     """Background Token Dropping.  Returns (idx [capacity] i32, n_out [1] i32, outs)."""
     T = mask.shape[0]
-    row_bytes = srcs[0][0].numel() * srcs[0].element_size() if T else 16
+    row_bytes = _row_bytes(srcs, T, "srcs")
     cap = T if capacity is None else int(capacity)
     dev = mask.device
     if outs is None:
         outs = [torch.empty((cap,) + tuple(s.shape[1:]), dtype=s.dtype, device=dev) for s in srcs]
+    if len(outs) != len(srcs) or _row_bytes(outs, cap, "outs") != row_bytes:
+        raise ValueError("outs must match srcs row for row")
+    if idx is not None and idx.numel() < cap:
+        raise ValueError("idx holds fewer than capacity entries")
     if idx is None:
         idx = torch.empty(max(cap, 1), dtype=torch.int32, device=dev)
     if n_out is None:
@@ -155,7 +180,13 @@ def ut_fg_scatter(idx: torch.Tensor, n: int, srcs: Sequence[torch.Tensor], dsts:
                   bg_mode: int = UT_BG_KEEP, fill_row: Optional[torch.Tensor] = None) -> None:
     """dst[idx[i]] = src[i] for i < n; background rows per bg_mode."""
     T = dsts[0].shape[0]
-    row_bytes = dsts[0][0].numel() * dsts[0].element_size()
+    row_bytes = _row_bytes(dsts, T, "dsts")
+    if len(srcs) != len(dsts) or _row_bytes(srcs, int(n), "srcs") != row_bytes:
+        raise ValueError("srcs must match dsts row for row")
+    if fill_row is not None and fill_row.numel() * fill_row.element_size() != row_bytes:
+        raise ValueError("fill_row must hold exactly one row")
+    if idx.numel() < int(n):
+        raise ValueError("idx holds fewer than n entries")
     st = lib().ut_fg_scatter(_p(idx), int(n), len(srcs), _ptr_array(srcs), _ptr_array(dsts), row_bytes, bg_mode,
                              _p(fill_row), T, _stream())
     _check("ut_fg_scatter", st)

@@ -101,3 +101,19 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(u, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="missing"):
         u.lib()
+
+
+def test_binding_rejects_mixed_row_sizes():
+    """One row size per call: a list mixing row sizes never reaches a kernel."""
+    import torch
+    from paper_2609_23169_gb300 import ultratex as u
+    m = torch.ones(10, dtype=torch.uint8)
+    a = torch.zeros(10, 2, 128, dtype=torch.bfloat16)
+    b = torch.zeros(10, 8, dtype=torch.float32)
+    with pytest.raises(ValueError, match="row size"):
+        u.ut_fg_compact(m, [a, b])
+    with pytest.raises(ValueError, match="rows"):
+        u.ut_fg_compact(m, [a[:5]])
+    idx = torch.zeros(10, dtype=torch.int32)
+    with pytest.raises(ValueError):
+        u.ut_fg_scatter(idx, 10, [a], [b])
