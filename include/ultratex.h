@@ -16,7 +16,8 @@
  *   - Pointers are DEVICE pointers unless the parameter name starts with h_
  *     (host memory).  The caller owns every buffer, including workspaces
  *     sized by the *_workspace_size functions.  No entry point allocates or
- *     frees memory, synchronises the device or keeps global state.
+ *     frees memory, synchronises the device or keeps global state (the one
+ *     exception to the last, ut_fg_compact_noalloc, says so below).
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy stream).  All
  *     work is enqueued on it; results are valid once the stream has reached
  *     the enqueued work.
@@ -100,6 +101,23 @@ ut_status ut_fg_compact(const uint8_t* mask, int64_t T, int32_t n_tensors,
                         const void* const* h_src, void* const* h_dst, int64_t row_bytes,
                         int64_t capacity, int32_t* idx_out, int32_t* n_out,
                         void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
+
+/* ut_fg_compact without a caller workspace.  The paper has no counterpart:
+ * this entry point exists for callers that cannot allocate device memory
+ * (a host that owns every allocation and passes the library only its inputs
+ * and outputs, or a loop that must not enter an allocator).  Same arguments
+ * and results as ut_fg_compact, minus ws / ws_bytes.  Its scratch is a fixed
+ * 4 KiB device array inside the library (held by every GPU that loads it
+ * until exit), so T is limited to 4,194,304 canvas tokens; a larger T
+ * returns UT_ERR_UNSUPPORTED before anything is enqueued.  The first call on
+ * a device looks up the array's address with that device current; make it
+ * before any stream capture.  All calls share the array: calls that overlap
+ * on the GPU race and must be serialised by the caller.  No allocation,
+ * free or allocating library routine is called. */
+ut_status ut_fg_compact_noalloc(const uint8_t* mask, int64_t T, int32_t n_tensors,
+                                const void* const* h_src, void* const* h_dst, int64_t row_bytes,
+                                int64_t capacity, int32_t* idx_out, int32_t* n_out,
+                                int32_t* dev_status, void* stream);
 
 /* ------------------------------------------------------------------------
  * Scatter compacted rows back to the canvas: dst[idx[n]] = src[n] for n < N.

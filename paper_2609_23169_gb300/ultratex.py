@@ -24,7 +24,7 @@ UT_MASK_TOPK, UT_MASK_BITMAP = 0, 1
 EXPORTS = (
     "ut_strerror", "ut_topk_count", "ut_fg_compact_workspace_size", "ut_fg_compact", "ut_fg_scatter",
     "ut_block_mask_workspace_size", "ut_block_mask", "ut_bsattn_fwd", "ut_bsattn_bwd_workspace_size",
-    "ut_bsattn_bwd",
+    "ut_bsattn_bwd", "ut_fg_compact_noalloc",
 )
 
 
