@@ -94,11 +94,18 @@ struct DqSmem {
   alignas(1024) uint8_t v[2][kTileBytes];
   alignas(1024) uint8_t ds[kTile * kTile * 2];
   uint64_t qd_full, qd_empty;
-  uint64_t k_full[2], v_full[2], kv_empty[2];
-  uint64_t sp_full, sp_empty, ds_full, dq_mma_done, dq_empty, mma_done;
+  uint64_t k_full[2], v_full[2], k_empty[2], v_empty[2];
+  uint64_t s_full, s_empty, dp_full, dp_empty, ds_full, dq_mma_done, dq_empty, mma_done;
   uint32_t tmem_base;
   int abort_flag;
 };
+
+// 64 consecutive TMEM columns of this warp's 32 lanes, one wait.
+UT_DEV void tmem_ld64(uint32_t taddr, uint32_t* r) {
+  tmem_ld32(taddr, *reinterpret_cast<uint32_t(*)[32]>(r));
+  tmem_ld32(taddr + 32, *reinterpret_cast<uint32_t(*)[32]>(r + 32));
+  tmem_wait_ld();
+}
 
 template <int D>
 __global__ void __launch_bounds__(kBwdThreads, 1)
@@ -121,10 +128,13 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.k_full[s], 1);
       mbar_init(&sm.v_full[s], 1);
-      mbar_init(&sm.kv_empty[s], 1);
+      mbar_init(&sm.k_empty[s], 1);
+      mbar_init(&sm.v_empty[s], 1);
     }
-    mbar_init(&sm.sp_full, 1);
-    mbar_init(&sm.sp_empty, 4);
+    mbar_init(&sm.s_full, 1);
+    mbar_init(&sm.s_empty, 4);
+    mbar_init(&sm.dp_full, 1);
+    mbar_init(&sm.dp_empty, 4);
     mbar_init(&sm.ds_full, 4);
     mbar_init(&sm.dq_mma_done, 1);
     mbar_init(&sm.dq_empty, 4);
@@ -143,36 +153,45 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   const int G = gridDim.x;
 
   if (warp == 0) {
-    if (lane == 0) {
-      tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
-      tma_prefetch_desc(&tm_do);
+    // lane 0: Q, dO and the K ring (K is freed after dQ += dS K);
+    // lane 1: the V ring (V is freed after dP = dO V^T).
+    if (lane < 2) {
+      const bool is_k = lane == 0;
+      if (is_k) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+        tma_prefetch_desc(&tm_do);
+      } else {
+        tma_prefetch_desc(&tm_v);
+      }
       const uint64_t pol_kv = policy_evict_last(), pol_q = policy_evict_first();
+      uint64_t* full = is_k ? sm.k_full : sm.v_full;
+      uint64_t* empty = is_k ? sm.k_empty : sm.v_empty;
+      uint8_t* ring = is_k ? &sm.k[0][0] : &sm.v[0][0];
+      const void* tmap = is_k ? static_cast<const void*>(&tm_k) : static_cast<const void*>(&tm_v);
       uint32_t qi = 0, kv = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int h = w / prm.nq, i = w % prm.nq;
         const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
         if (L <= 0) continue;
-        if (!(ok = mbar_wait(&sm.qd_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        mbar_expect_tx(&sm.qd_full, 2 * TB);
-        for (int c = 0; c < C; ++c) {
-          tma_load_2d(sm.q + c * kChunk, &tm_q, &sm.qd_full, h * D + c * 64, i * kTile, pol_q);
-          tma_load_2d(sm.dout + c * kChunk, &tm_do, &sm.qd_full, h * D + c * 64, i * kTile, pol_q);
+        if (is_k) {
+          if (!(ok = mbar_wait(&sm.qd_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&sm.qd_full, 2 * TB);
+          for (int c = 0; c < C; ++c) {
+            tma_load_2d(sm.q + c * kChunk, &tm_q, &sm.qd_full, h * D + c * 64, i * kTile, pol_q);
+            tma_load_2d(sm.dout + c * kChunk, &tm_do, &sm.qd_full, h * D + c * 64, i * kTile, pol_q);
+          }
+          ++qi;
         }
-        ++qi;
         for (int t = 0; t < L; ++t, ++kv) {
           const int j = prm.idx[beg + t];
           const int st = kv & 1;
           const uint32_t n = kv >> 1;
-          if (!(ok = mbar_wait(&sm.kv_empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          mbar_expect_tx(&sm.k_full[st], TB);
+          if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&full[st], TB);
           for (int c = 0; c < C; ++c)
-            tma_load_2d(sm.k[st] + c * kChunk, &tm_k, &sm.k_full[st], h * D + c * 64, j * kTile, pol_kv);
-          mbar_expect_tx(&sm.v_full[st], TB);
-          for (int c = 0; c < C; ++c)
-            tma_load_2d(sm.v[st] + c * kChunk, &tm_v, &sm.v_full[st], h * D + c * 64, j * kTile, pol_kv);
+            tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, j * kTile, pol_kv);
         }
       }
       const uint64_t t0 = globaltimer();
@@ -181,10 +200,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
       };
       if (qi > 0) drain(&sm.qd_full, (qi - 1) & 1);
-      for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) {
-        drain(&sm.k_full[u & 1], (u >> 1) & 1);
-        drain(&sm.v_full[u & 1], (u >> 1) & 1);
-      }
+      for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) drain(&full[u & 1], (u >> 1) & 1);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -201,24 +217,29 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           if (t < L) {
             const uint32_t kv = kv0 + t, st = kv & 1, n = kv >> 1;
             const uint32_t sc = sc0 + t;
-            if (!(ok = mbar_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.sp_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            tc_fence_after();
+            // S = Q K^T once the previous S has been read; dP = dO V^T once the previous dP has
             const uint32_t k_addr = smem_u32(sm.k[st]), v_addr = smem_u32(sm.v[st]);
+            if (!(ok = mbar_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.s_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
               mma_bf16_ss(tmem, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024), idesc_s,
                           kk > 0);
             }
+            mma_commit(&sm.s_full);
+            if (!(ok = mbar_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.dp_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
               mma_bf16_ss(tmem + 128, sdesc_sw128(do_addr + off, 16, 1024), sdesc_sw128(v_addr + off, 16, 1024),
                           idesc_s, kk > 0);
             }
-            mma_commit(&sm.sp_full);
+            mma_commit(&sm.dp_full);
+            mma_commit(&sm.v_empty[st]);
             if (t == L - 1) mma_commit(&sm.qd_empty);
           }
           if (t >= 1) {
@@ -237,7 +258,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
                           sdesc_sw128(k_addr + kk * 2048, kChunk, 1024), idesc_dq, (u > 0 || kk > 0));
             }
             mma_commit(&sm.dq_mma_done);
-            mma_commit(&sm.kv_empty[st]);
+            mma_commit(&sm.k_empty[st]);
           }
         }
         kv0 += L;
@@ -269,54 +290,58 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       }
       const float lse2 = prm.lse2[(int64_t)h * prm.Np + grow];
       const float Dr = prm.dsum[(int64_t)h * prm.Np + grow];
+      int j_cur = prm.idx[beg];
       for (int t = 0; t < L; ++t) {
         const uint32_t sc = sc0 + t;
-        if (!(ok = warp_wait(&sm.sp_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        tc_fence_after();
-        const int j = prm.idx[beg + t];
+        const int j = j_cur;
+        if (t + 1 < L) j_cur = prm.idx[beg + t + 1];  // prefetch the next key block index
         const int64_t nv = prm.N - (int64_t)j * kTile;
+        if (!(ok = warp_wait(&sm.s_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
         float p[kTile];
+        {
+          uint32_t r[kTile];
 #pragma unroll
-        for (int g = 0; g < kTile / 32; ++g) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_base + g * 32, r);
+          for (int g = 0; g < kTile / 32; ++g)
+            tmem_ld32(tmem + lane_base + g * 32, *reinterpret_cast<uint32_t(*)[32]>(&r[g * 32]));
           tmem_wait_ld();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.s_empty);
 #pragma unroll
-          for (int x = 0; x < 32; ++x) {
-            const int col = g * 32 + x;
-            p[col] = col < nv ? ex2_approx(fmaf(__uint_as_float(r[x]), c, -lse2)) : 0.f;
-          }
+          for (int col = 0; col < kTile; ++col)
+            p[col] = col < nv ? ex2_approx(fmaf(__uint_as_float(r[col]), c, -lse2)) : 0.f;
         }
+        if (!(ok = warp_wait(&sm.dp_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
         // dS buffer is free once the previous tile's dQ MMA finished
         if (!(ok = warp_wait(&sm.dq_mma_done, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
         const uint32_t ds_row = smem_u32(sm.ds) + row * 128;
 #pragma unroll
-        for (int g = 0; g < kTile / 32; ++g) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_base + 128 + g * 32, r);
-          tmem_wait_ld();
-          uint32_t pk[16];
-#pragma unroll
-          for (int x = 0; x < 32; x += 2) {
-            const float d0 = p[g * 32 + x] * (__uint_as_float(r[x]) - Dr);
-            const float d1 = p[g * 32 + x + 1] * (__uint_as_float(r[x + 1]) - Dr);
-            pk[x / 2] = pack_bf16x2(d0, d1);
+        for (int half = 0; half < 2; ++half) {
+          uint32_t r[64];
+          tmem_ld64(tmem + lane_base + 128 + half * 64, r);
+          if (half == 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.dp_empty);
           }
 #pragma unroll
-          for (int u4 = 0; u4 < 4; ++u4) {
-            const uint32_t u = g * 4 + u4;  // 16-byte unit (8 keys) within the 128-key row
+          for (int u8 = 0; u8 < 8; ++u8) {
+            const int col = half * 64 + u8 * 8;
+            uint32_t pk[4];
+#pragma unroll
+            for (int x = 0; x < 8; x += 2)
+              pk[x / 2] = pack_bf16x2(p[col + x] * (__uint_as_float(r[u8 * 8 + x]) - Dr),
+                                      p[col + x + 1] * (__uint_as_float(r[u8 * 8 + x + 1]) - Dr));
+            const uint32_t u = half * 8 + u8;  // 16-byte unit (8 keys) within the 128-key row
             const uint32_t chunk = u >> 3, unit = u & 7;
-            st_shared_v4(ds_row + chunk * kChunk + ((unit ^ (row & 7)) << 4), pk[4 * u4], pk[4 * u4 + 1],
-                         pk[4 * u4 + 2], pk[4 * u4 + 3]);
+            st_shared_v4(ds_row + chunk * kChunk + ((unit ^ (row & 7)) << 4), pk[0], pk[1], pk[2], pk[3]);
           }
         }
-        tc_fence_before();
         fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&sm.sp_empty);
-          mbar_arrive(&sm.ds_full);
-        }
+        if (lane == 0) mbar_arrive(&sm.ds_full);
       }
       if (!ok) break;
       const uint32_t last = sc0 + L - 1;
@@ -363,11 +388,11 @@ struct DkdvSmem {
   alignas(1024) uint8_t q[2][kTileBytes];
   alignas(1024) uint8_t dout[2][kTileBytes];
   alignas(1024) uint8_t pds[kTile * kTile * 2];   // P^T, then dS^T, of the current pair
-  float lse2[2][kTile];
-  float dsum[2][kTile];
+  alignas(16) float lse2[2][kTile];
+  alignas(16) float dsum[2][kTile];
   uint64_t kv_full, kv_empty;
-  uint64_t qd_full[2], qd_empty[2];
-  uint64_t sp_full, sp_empty, pt_full, pt_done, dst_full, ds_done, acc_full, acc_empty, mma_done;
+  uint64_t q_full[2], q_empty[2], do_full[2], do_empty[2];
+  uint64_t s_full, s_empty, dp_full, dp_empty, pt_full, pt_done, dst_full, ds_done, acc_full, acc_empty, mma_done;
   uint64_t rowvec_full[2];   // the 128 elementwise threads staged this pair's LSE / D
   uint32_t tmem_base;
   int abort_flag;
@@ -392,11 +417,15 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     mbar_init(&sm.kv_full, 1);
     mbar_init(&sm.kv_empty, 1);
     for (int s = 0; s < 2; ++s) {
-      mbar_init(&sm.qd_full[s], 1);
-      mbar_init(&sm.qd_empty[s], 1);
+      mbar_init(&sm.q_full[s], 1);
+      mbar_init(&sm.q_empty[s], 1);
+      mbar_init(&sm.do_full[s], 1);
+      mbar_init(&sm.do_empty[s], 1);
     }
-    mbar_init(&sm.sp_full, 1);
-    mbar_init(&sm.sp_empty, 4);
+    mbar_init(&sm.s_full, 1);
+    mbar_init(&sm.s_empty, 4);
+    mbar_init(&sm.dp_full, 1);
+    mbar_init(&sm.dp_empty, 4);
     mbar_init(&sm.pt_full, 4);
     mbar_init(&sm.pt_done, 1);
     mbar_init(&sm.dst_full, 4);
@@ -420,35 +449,45 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   const int G = gridDim.x;
 
   if (warp == 0) {
-    if (lane == 0) {
-      tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
-      tma_prefetch_desc(&tm_do);
+    // lane 0: K, V of the item and the Q ring (Q is freed after dK += dS^T Q);
+    // lane 1: the dO ring (dO is freed after dV += P^T dO).
+    if (lane < 2) {
+      const bool is_q = lane == 0;
+      if (is_q) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+        tma_prefetch_desc(&tm_v);
+      } else {
+        tma_prefetch_desc(&tm_do);
+      }
       const uint64_t pol_qd = policy_evict_last(), pol_kv = policy_evict_first();
+      uint64_t* full = is_q ? sm.q_full : sm.do_full;
+      uint64_t* empty = is_q ? sm.q_empty : sm.do_empty;
+      uint8_t* ring = is_q ? &sm.q[0][0] : &sm.dout[0][0];
+      const void* tmap = is_q ? static_cast<const void*>(&tm_q) : static_cast<const void*>(&tm_do);
       uint32_t ki = 0, qd = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int h = w / prm.nq, j = w % prm.nq;
         const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
         if (L <= 0) continue;
-        if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        mbar_expect_tx(&sm.kv_full, 2 * TB);
-        for (int c = 0; c < C; ++c) {
-          tma_load_2d(sm.k + c * kChunk, &tm_k, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
-          tma_load_2d(sm.v + c * kChunk, &tm_v, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
+        if (is_q) {
+          if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&sm.kv_full, 2 * TB);
+          for (int c = 0; c < C; ++c) {
+            tma_load_2d(sm.k + c * kChunk, &tm_k, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
+            tma_load_2d(sm.v + c * kChunk, &tm_v, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
+          }
+          ++ki;
         }
-        ++ki;
         for (int t = 0; t < L; ++t, ++qd) {
           const int i = prm.idx[beg + t];
           const int st = qd & 1;
           const uint32_t n = qd >> 1;
-          if (!(ok = mbar_wait(&sm.qd_empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          mbar_expect_tx(&sm.qd_full[st], 2 * TB);
-          for (int c = 0; c < C; ++c) {
-            tma_load_2d(sm.q[st] + c * kChunk, &tm_q, &sm.qd_full[st], h * D + c * 64, i * kTile, pol_qd);
-            tma_load_2d(sm.dout[st] + c * kChunk, &tm_do, &sm.qd_full[st], h * D + c * 64, i * kTile, pol_qd);
-          }
+          if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&full[st], TB);
+          for (int c = 0; c < C; ++c)
+            tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, i * kTile, pol_qd);
         }
       }
       const uint64_t t0 = globaltimer();
@@ -457,7 +496,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
       };
       if (ki > 0) drain(&sm.kv_full, (ki - 1) & 1);
-      for (uint32_t u = (qd >= 2 ? qd - 2 : 0); u < qd; ++u) drain(&sm.qd_full[u & 1], (u >> 1) & 1);
+      for (uint32_t u = (qd >= 2 ? qd - 2 : 0); u < qd; ++u) drain(&full[u & 1], (u >> 1) & 1);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -471,31 +510,25 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         if (L <= 0) continue;
         if (!(ok = mbar_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         for (int t = 0; t <= L && ok; ++t) {
+          // issue order per step: S^T_t, dV_{t-1}, dP^T_t, dK_{t-1}
+          const uint32_t qd_t = qd0 + t, st_t = qd_t & 1, n_t = qd_t >> 1;
           if (t < L) {
-            const uint32_t qd = qd0 + t, st = qd & 1, n = qd >> 1;
-            if (!(ok = mbar_wait(&sm.qd_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.sp_empty, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.q_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.s_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
-            const uint32_t q_addr = smem_u32(sm.q[st]), do_addr = smem_u32(sm.dout[st]);
+            const uint32_t q_addr = smem_u32(sm.q[st_t]);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
               mma_bf16_ss(tmem, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024), idesc_s,
                           kk > 0);
             }
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss(tmem + 128, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
-                          idesc_s, kk > 0);
-            }
-            mma_commit(&sm.sp_full);
-            if (t == L - 1) mma_commit(&sm.kv_empty);
+            mma_commit(&sm.s_full);
           }
           if (t >= 1) {
             const uint32_t u = t - 1;
             const uint32_t qd = qd0 + u, st = qd & 1;
-            const uint32_t q_addr = smem_u32(sm.q[st]), do_addr = smem_u32(sm.dout[st]);
+            const uint32_t do_addr = smem_u32(sm.dout[st]);
             if (!(ok = mbar_wait(&sm.pt_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             if (u == 0 && !(ok = mbar_wait(&sm.acc_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
               break;
@@ -507,6 +540,26 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
                           sdesc_sw128(do_addr + kk * 2048, kChunk, 1024), idesc_acc, (u > 0 || kk > 0));
             }
             mma_commit(&sm.pt_done);
+            mma_commit(&sm.do_empty[st]);
+          }
+          if (t < L) {
+            if (!(ok = mbar_wait(&sm.do_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = mbar_wait(&sm.dp_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+            const uint32_t do_addr = smem_u32(sm.dout[st_t]);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss(tmem + 128, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
+                          idesc_s, kk > 0);
+            }
+            mma_commit(&sm.dp_full);
+            if (t == L - 1) mma_commit(&sm.kv_empty);
+          }
+          if (t >= 1) {
+            const uint32_t u = t - 1;
+            const uint32_t qd = qd0 + u, st = qd & 1;
+            const uint32_t q_addr = smem_u32(sm.q[st]);
             if (!(ok = mbar_wait(&sm.dst_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
 #pragma unroll
@@ -516,7 +569,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
                           sdesc_sw128(q_addr + kk * 2048, kChunk, 1024), idesc_acc, (u > 0 || kk > 0));
             }
             mma_commit(&sm.ds_done);
-            mma_commit(&sm.qd_empty[st]);
+            mma_commit(&sm.q_empty[st]);
           }
         }
         mma_commit(&sm.acc_full);
@@ -564,16 +617,26 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           break;
         const float* ls = sm.lse2[qd & 1];
         const float* ds_v = sm.dsum[qd & 1];
-        if (!(ok = warp_wait(&sm.sp_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        if (!(ok = warp_wait(&sm.s_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
         float p[kTile];
+        {
+          uint32_t r[kTile];
 #pragma unroll
-        for (int g = 0; g < kTile / 32; ++g) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_base + g * 32, r);
+          for (int g = 0; g < kTile / 32; ++g)
+            tmem_ld32(tmem + lane_base + g * 32, *reinterpret_cast<uint32_t(*)[32]>(&r[g * 32]));
           tmem_wait_ld();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.s_empty);
 #pragma unroll
-          for (int x = 0; x < 32; ++x) p[g * 32 + x] = ex2_approx(fmaf(__uint_as_float(r[x]), c, -ls[g * 32 + x]));
+          for (int x = 0; x < kTile; x += 4) {
+            const float4 l4 = *reinterpret_cast<const float4*>(ls + x);
+            p[x + 0] = ex2_approx(fmaf(__uint_as_float(r[x + 0]), c, -l4.x));
+            p[x + 1] = ex2_approx(fmaf(__uint_as_float(r[x + 1]), c, -l4.y));
+            p[x + 2] = ex2_approx(fmaf(__uint_as_float(r[x + 2]), c, -l4.z));
+            p[x + 3] = ex2_approx(fmaf(__uint_as_float(r[x + 3]), c, -l4.w));
+          }
         }
         // the shared P/dS tile is free once the previous pair's dK MMA finished
         if (!(ok = warp_wait(&sm.ds_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -589,21 +652,27 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.pt_full);
         uint32_t dsk[kTile / 2];
+        if (!(ok = warp_wait(&sm.dp_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
 #pragma unroll
-        for (int g = 0; g < kTile / 32; ++g) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_base + 128 + g * 32, r);
-          tmem_wait_ld();
+        for (int half = 0; half < 2; ++half) {
+          uint32_t r[64];
+          tmem_ld64(tmem + lane_base + 128 + half * 64, r);
+          if (half == 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.dp_empty);
+          }
 #pragma unroll
-          for (int x = 0; x < 32; x += 2) {
-            const int col = g * 32 + x;
-            dsk[col / 2] = pack_bf16x2(p[col] * (__uint_as_float(r[x]) - ds_v[col]),
-                                       p[col + 1] * (__uint_as_float(r[x + 1]) - ds_v[col + 1]));
+          for (int x = 0; x < 64; x += 4) {
+            const int col = half * 64 + x;
+            const float4 d4 = *reinterpret_cast<const float4*>(ds_v + col);
+            dsk[col / 2] = pack_bf16x2(p[col] * (__uint_as_float(r[x]) - d4.x),
+                                       p[col + 1] * (__uint_as_float(r[x + 1]) - d4.y));
+            dsk[col / 2 + 1] = pack_bf16x2(p[col + 2] * (__uint_as_float(r[x + 2]) - d4.z),
+                                           p[col + 3] * (__uint_as_float(r[x + 3]) - d4.w));
           }
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.sp_empty);
         // overwrite P^T with dS^T once the dV MMA has read P^T
         if (!(ok = warp_wait(&sm.pt_done, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
 #pragma unroll
@@ -659,6 +728,10 @@ size_t attn_bwd_tc_ws(const AttnProblem& p) {
   const size_t Np = (size_t)p.nq * kTile;
   return 2 * (size_t)p.H * Np * sizeof(float);
 }
+
+constexpr size_t kMaxDynSmem = 232448;  // 227 KB opt-in per block on sm_100/sm_103
+static_assert(sizeof(DqSmem<128>) <= kMaxDynSmem, "dQ shared layout exceeds the per-block limit");
+static_assert(sizeof(DkdvSmem<128>) <= kMaxDynSmem, "dK/dV shared layout exceeds the per-block limit");
 
 template <int D>
 static cudaError_t launch_bwd_d(const AttnProblem& p, const CUtensorMap* tm, BwdParams prm_dq, BwdParams prm_kv,

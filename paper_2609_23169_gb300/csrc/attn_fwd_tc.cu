@@ -39,7 +39,7 @@ struct FwdSmem {
   alignas(1024) uint8_t v[2][kKVBytes];
   alignas(1024) uint8_t p[2][kPBytes];
   uint64_t q_full, q_empty;
-  uint64_t k_full[2], v_full[2], kv_empty[2];
+  uint64_t k_full[2], v_full[2], k_empty[2], v_empty[2];
   uint64_t s_full[2], s_empty[2];
   uint64_t p_full[2], pv_done[2];
   uint64_t o_empty, mma_done;
@@ -78,7 +78,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.k_full[s], 1);
       mbar_init(&sm.v_full[s], 1);
-      mbar_init(&sm.kv_empty[s], 1);
+      mbar_init(&sm.k_empty[s], 1);
+      mbar_init(&sm.v_empty[s], 1);
       mbar_init(&sm.s_full[s], 1);
       mbar_init(&sm.s_empty[s], 4);
       mbar_init(&sm.p_full[s], 4);
@@ -101,47 +102,55 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   const int G = gridDim.x;
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
+    // lane 0 streams Q and K, lane 1 streams V: each ring is released by the
+    // MMA that consumes it (K after S = Q K^T, V after O += P V), so neither
+    // waits for the other.
+    if (lane < 2) {
+      const bool is_k = lane == 0;
+      if (is_k) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+      } else {
+        tma_prefetch_desc(&tm_v);
+      }
       const uint64_t pol_kv = policy_evict_last();
       const uint64_t pol_q = policy_evict_first();
+      uint64_t* full = is_k ? sm.k_full : sm.v_full;
+      uint64_t* empty = is_k ? sm.k_empty : sm.v_empty;
+      uint8_t* ring = is_k ? &sm.k[0][0] : &sm.v[0][0];
+      const void* tmap = is_k ? static_cast<const void*>(&tm_k) : static_cast<const void*>(&tm_v);
       uint32_t qi = 0, kv = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int h = w / prm.nq, i = w % prm.nq;
         const int beg = prm.row_ptr[w], L = prm.row_ptr[w + 1] - beg;
         if (L <= 0) continue;
-        if (!(ok = mbar_wait(&sm.q_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        mbar_expect_tx(&sm.q_full, FwdSmem<D>::kQBytes);
-        for (int c = 0; c < C; ++c)
-          tma_load_2d(sm.q + c * kTileChunkBytes, &tm_q, &sm.q_full, h * D + c * 64, i * kBM, pol_q);
-        ++qi;
+        if (is_k) {
+          if (!(ok = mbar_wait(&sm.q_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&sm.q_full, FwdSmem<D>::kQBytes);
+          for (int c = 0; c < C; ++c)
+            tma_load_2d(sm.q + c * kTileChunkBytes, &tm_q, &sm.q_full, h * D + c * 64, i * kBM, pol_q);
+          ++qi;
+        }
         for (int t = 0; t < L; ++t, ++kv) {
           const int j = prm.col_idx[beg + t];
           const int st = kv & 1;
           const uint32_t n = kv >> 1;
-          if (!(ok = mbar_wait(&sm.kv_empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          mbar_expect_tx(&sm.k_full[st], FwdSmem<D>::kKVBytes);
+          if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          mbar_expect_tx(&full[st], FwdSmem<D>::kKVBytes);
           for (int c = 0; c < C; ++c)
-            tma_load_2d(sm.k[st] + c * kTileChunkBytes, &tm_k, &sm.k_full[st], h * D + c * 64, j * kBN, pol_kv);
-          mbar_expect_tx(&sm.v_full[st], FwdSmem<D>::kKVBytes);
-          for (int c = 0; c < C; ++c)
-            tma_load_2d(sm.v[st] + c * kTileChunkBytes, &tm_v, &sm.v_full[st], h * D + c * 64, j * kBN, pol_kv);
+            tma_load_2d(ring + st * FwdSmem<D>::kKVBytes + c * kTileChunkBytes, tmap, &full[st], h * D + c * 64,
+                        j * kBN, pol_kv);
         }
       }
-      // Drain: every issued copy has landed before the CTA may exit.
+      // Drain: every copy this lane issued has landed before the CTA may exit.
       const uint64_t t0 = globaltimer();
       auto drain = [&](uint64_t* bar, uint32_t parity) {
         while (!mbar_try_wait(bar, parity))
           if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
       };
       if (qi > 0) drain(&sm.q_full, (qi - 1) & 1);
-      for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) {
-        drain(&sm.k_full[u & 1], (u >> 1) & 1);
-        drain(&sm.v_full[u & 1], (u >> 1) & 1);
-      }
+      for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) drain(&full[u & 1], (u >> 1) & 1);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------- MMA issuer
@@ -170,6 +179,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
                           idesc_s, kk > 0);
             }
             mma_commit(&sm.s_full[sb]);
+            mma_commit(&sm.k_empty[st]);
             if (t == L - 1) mma_commit(&sm.q_empty);
           }
           if (t >= 1) {
@@ -190,7 +200,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
                           sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024), idesc_o, (u > 0 || kk > 0));
             }
             mma_commit(&sm.pv_done[pb]);
-            mma_commit(&sm.kv_empty[st]);
+            mma_commit(&sm.v_empty[st]);
           }
         }
         kv0 += L;
@@ -226,33 +236,40 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         continue;
       }
       float m_used = 0.f, l = 0.f;
+      int j_cur = prm.col_idx[beg];
       for (int t = 0; t < L; ++t) {
         const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
         if (!(ok = warp_wait(&sm.s_full[sb], ns & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
-        float s[kBN];
+        // all four 32-column loads in flight before one wait
+        uint32_t r[kBN];
 #pragma unroll
-        for (int g = 0; g < kBN / 32; ++g) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_base + sb * 128 + g * 32, r);
-          tmem_wait_ld();
-#pragma unroll
-          for (int x = 0; x < 32; ++x) s[g * 32 + x] = __uint_as_float(r[x]);
-        }
+        for (int g = 0; g < kBN / 32; ++g)
+          tmem_ld32(tmem + lane_base + sb * 128 + g * 32, *reinterpret_cast<uint32_t(*)[32]>(&r[g * 32]));
+        tmem_wait_ld();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.s_empty[sb]);
+        float s[kBN];
+#pragma unroll
+        for (int x = 0; x < kBN; ++x) s[x] = __uint_as_float(r[x]);
         // ragged last key block: columns past N do not exist
-        const int j = prm.col_idx[beg + t];
+        const int j = j_cur;
+        if (t + 1 < L) j_cur = prm.col_idx[beg + t + 1];  // prefetch the next block index
         const int64_t nv = prm.N - (int64_t)j * kBN;
         if (nv < kBN) {
 #pragma unroll
           for (int x = 0; x < kBN; ++x)
             if (x >= nv) s[x] = -INFINITY;
         }
-        float mx = s[0];
+        // row maximum as a tree (8 independent chains) rather than one long chain
+        float m8[8];
 #pragma unroll
-        for (int x = 1; x < kBN; ++x) mx = fmaxf(mx, s[x]);
+        for (int q = 0; q < 8; ++q) m8[q] = s[q];
+#pragma unroll
+        for (int x = 8; x < kBN; ++x) m8[x & 7] = fmaxf(m8[x & 7], s[x]);
+        float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                         fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
         mx *= c;
         if (t == 0) {
           m_used = mx;
@@ -282,15 +299,15 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         }
         // P = exp2(s * c - m_used), rounded to bf16 for the P V MMA
         uint32_t pk[kBN / 2];
-        float lsum = 0.f;
+        float l8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int x = 0; x < kBN; x += 2) {
           const float p0 = ex2_approx(fmaf(s[x], c, -m_used));
           const float p1 = ex2_approx(fmaf(s[x + 1], c, -m_used));
-          lsum += p0 + p1;
+          l8[(x >> 1) & 7] += p0 + p1;
           pk[x / 2] = pack_bf16x2(p0, p1);
         }
-        l += lsum;
+        l += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
         // the P buffer is free once the P V MMA of its previous use finished
         if (!(ok = warp_wait(&sm.pv_done[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
         const uint32_t p_row = smem_u32(sm.p[sb]) + row * 128;
@@ -341,6 +358,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, 512);
 }
+
+static_assert(sizeof(FwdSmem<128>) + 1024 <= 232448, "forward shared layout exceeds the per-block limit");
 
 template <int D>
 static cudaError_t launch_d(const AttnProblem& p, const CUtensorMap& tq, const CUtensorMap& tk,
