@@ -4,18 +4,21 @@
 //
 // Persistent kernel, one CTA per SM, work items (h, i) in head-major order so
 // that the CTAs in flight share one head's K/V in L2.  Roles (192 threads):
-//   warp 0      TMA producer: Q tile of the item, then K_j / V_j of every
-//               listed key block into a 2-stage ring (128B-swizzled tiles).
+//   warp 0      TMA producers: lane 0 streams the item's Q tile and the K tiles,
+//               lane 1 the V tiles, each into its own 3-stage ring of
+//               128B-swizzled shared tiles.  A K stage is released by the MMA
+//               that consumed it (S = Q K^T), a V stage by O += P V.
 //   warp 1      TMEM owner and MMA issuer (one elected thread):
-//               S_t = Q K_t^T into one of two TMEM S buffers, then
-//               O += P_{t-1} V_{t-1} into the TMEM O accumulator.
+//               S_t = Q K_t^T (both operands in shared memory) into one of two
+//               TMEM S buffers, then O += P_{t-1} V_{t-1} with P read from TMEM
+//               (only V is read from shared memory).
 //   warps 2-5   softmax: thread = query row = TMEM lane.  Reads S_t from TMEM,
 //               masks the ragged last key block, keeps a running row maximum
 //               (rescaling O in TMEM only when the maximum grew by more than
-//               2^8, so the exponentials stay bounded), writes P_t as bf16 into
-//               a 128B-swizzled shared tile for the P V MMA, and finally
-//               normalises O, writes O (bf16) and LSE (fp32, natural log).
-// TMEM: S buffers at columns [0,128) and [128,256), O at [256, 256+D).
+//               2^8, so the exponentials stay bounded), writes P_t as bf16
+//               pairs into a TMEM P buffer, and finally normalises O and
+//               writes O (bf16) and LSE (fp32, natural log).
+// TMEM columns: S0 [0,128), S1 [128,256), O [256,256+D), P0 [384,448), P1 [448,512).
 // Every wait is bounded; on expiry the kernel records UT_ERR_TIMEOUT,
 // drains its own copies and MMAs, frees TMEM and returns.
 #include "common.cuh"
@@ -26,20 +29,20 @@ namespace ut {
 constexpr int kBM = 128;  // query rows per tile
 constexpr int kBN = 128;  // key rows per tile
 constexpr int kFwdThreads = 192;
+constexpr int kStages = 3;                       // K and V ring depth
 constexpr uint32_t kTileChunkBytes = 128 * 128;  // 128 rows x 128 bytes (64 bf16)
+constexpr uint32_t kColO = 256, kColP = 384;     // TMEM column bases
 
 template <int D>
 struct FwdSmem {
   static constexpr int kChunks = D / 64;
   static constexpr uint32_t kQBytes = kBM * D * 2;
   static constexpr uint32_t kKVBytes = kBN * D * 2;
-  static constexpr uint32_t kPBytes = kBM * kBN * 2;
   alignas(1024) uint8_t q[kQBytes];
-  alignas(1024) uint8_t k[2][kKVBytes];
-  alignas(1024) uint8_t v[2][kKVBytes];
-  alignas(1024) uint8_t p[2][kPBytes];
+  alignas(1024) uint8_t k[kStages][kKVBytes];
+  alignas(1024) uint8_t v[kStages][kKVBytes];
   uint64_t q_full, q_empty;
-  uint64_t k_full[2], v_full[2], k_empty[2], v_empty[2];
+  uint64_t k_full[kStages], v_full[kStages], k_empty[kStages], v_empty[kStages];
   uint64_t s_full[2], s_empty[2];
   uint64_t p_full[2], pv_done[2];
   uint64_t o_empty, mma_done;
@@ -75,11 +78,13 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(&sm.q_full, 1);
     mbar_init(&sm.q_empty, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.k_full[s], 1);
       mbar_init(&sm.v_full[s], 1);
       mbar_init(&sm.k_empty[s], 1);
       mbar_init(&sm.v_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.s_full[s], 1);
       mbar_init(&sm.s_empty[s], 4);
       mbar_init(&sm.p_full[s], 4);
@@ -134,8 +139,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         }
         for (int t = 0; t < L; ++t, ++kv) {
           const int j = prm.col_idx[beg + t];
-          const int st = kv & 1;
-          const uint32_t n = kv >> 1;
+          const uint32_t st = kv % kStages, n = kv / kStages;
           if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
           mbar_expect_tx(&full[st], FwdSmem<D>::kKVBytes);
           for (int c = 0; c < C; ++c)
@@ -150,7 +154,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
       };
       if (qi > 0) drain(&sm.q_full, (qi - 1) & 1);
-      for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) drain(&full[u & 1], (u >> 1) & 1);
+      for (uint32_t u = (kv >= kStages ? kv - kStages : 0); u < kv; ++u)
+        drain(&full[u % kStages], (u / kStages) & 1);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------- MMA issuer
@@ -166,7 +171,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         if (!(ok = mbar_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         for (int t = 0; t <= L && ok; ++t) {
           if (t < L) {
-            const uint32_t kv = kv0 + t, st = kv & 1, n = kv >> 1;
+            const uint32_t kv = kv0 + t, st = kv % kStages, n = kv / kStages;
             const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
             if (!(ok = mbar_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             if (!(ok = mbar_wait(&sm.s_empty[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -184,21 +189,18 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           }
           if (t >= 1) {
             const uint32_t u = t - 1;
-            const uint32_t kv = kv0 + u, st = kv & 1, n = kv >> 1;
+            const uint32_t kv = kv0 + u, st = kv % kStages, n = kv / kStages;
             const uint32_t sc = sc0 + u, pb = sc & 1, np = sc >> 1;
             if (!(ok = mbar_wait(&sm.p_full[pb], np & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             if (!(ok = mbar_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             if (u == 0 && !(ok = mbar_wait(&sm.o_empty, (oi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
               break;
             tc_fence_after();
-            const uint32_t p_addr = smem_u32(sm.p[pb]);
             const uint32_t v_addr = smem_u32(sm.v[st]);
 #pragma unroll
-            for (int kk = 0; kk < kBN / 16; ++kk) {
-              const uint32_t aoff = (kk >> 2) * kTileChunkBytes + (kk & 3) * 32;
-              mma_bf16_ss(tmem + 256, sdesc_sw128(p_addr + aoff, 16, 1024),
+            for (int kk = 0; kk < kBN / 16; ++kk)
+              mma_bf16_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
                           sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024), idesc_o, (u > 0 || kk > 0));
-            }
             mma_commit(&sm.pv_done[pb]);
             mma_commit(&sm.v_empty[st]);
           }
@@ -284,11 +286,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 #pragma unroll
             for (int g = 0; g < D / 32; ++g) {
               uint32_t r[32];
-              tmem_ld32(tmem + lane_base + 256 + g * 32, r);
+              tmem_ld32(tmem + lane_base + kColO + g * 32, r);
               tmem_wait_ld();
 #pragma unroll
               for (int x = 0; x < 32; ++x) r[x] = __float_as_uint(__uint_as_float(r[x]) * alpha);
-              tmem_st32(tmem + lane_base + 256 + g * 32, r);
+              tmem_st32(tmem + lane_base + kColO + g * 32, r);
             }
             tmem_wait_st();
             if (need) {
@@ -308,16 +310,12 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           pk[x / 2] = pack_bf16x2(p0, p1);
         }
         l += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
-        // the P buffer is free once the P V MMA of its previous use finished
+        // the TMEM P buffer is free once the P V MMA of its previous use finished
         if (!(ok = warp_wait(&sm.pv_done[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        const uint32_t p_row = smem_u32(sm.p[sb]) + row * 128;
-#pragma unroll
-        for (int u = 0; u < kBN / 8; ++u) {
-          const uint32_t chunk = u >> 3, unit = u & 7;
-          const uint32_t addr = p_row + chunk * kTileChunkBytes + ((unit ^ (row & 7)) << 4);
-          st_shared_v4(addr, pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-        }
-        fence_proxy_async_smem();
+        tc_fence_after();
+        tmem_st32(tmem + lane_base + kColP + sb * 64, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
+        tmem_st32(tmem + lane_base + kColP + sb * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[32]));
+        tmem_wait_st();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.p_full[sb]);
@@ -331,7 +329,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 #pragma unroll
       for (int g = 0; g < D / 32; ++g) {
         uint32_t r[32];
-        tmem_ld32(tmem + lane_base + 256 + g * 32, r);
+        tmem_ld32(tmem + lane_base + kColO + g * 32, r);
         tmem_wait_ld();
         if (row_ok) {
 #pragma unroll
