@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include "../../include/ultratex.h"
@@ -54,7 +55,18 @@ bool encode_tmap_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner_elem
 
 static ut_status from_cuda(cudaError_t e) { return e == cudaSuccess ? UT_OK : UT_ERR_CUDA; }
 
-static uint64_t wait_timeout_ns() { return 2000000000ull; }  // 2 s per bounded wait
+// Limit of every bounded device wait: 2 s, or UT_WAIT_TIMEOUT_NS from the
+// environment (read at each call; 0 = give up at the first wait that is not
+// already satisfied, which the failure-detection tests use).
+static uint64_t wait_timeout_ns() {
+  const char* e = getenv("UT_WAIT_TIMEOUT_NS");
+  if (e && *e) {
+    char* end = nullptr;
+    unsigned long long v = strtoull(e, &end, 10);
+    if (end && *end == '\0') return (uint64_t)v;
+  }
+  return 2000000000ull;
+}
 
 // Common checks of an attention shape.  nq_out gets ceil(N / block).
 static ut_status check_shape(const ut_attn_shape* s, int* nq_out) {

@@ -197,7 +197,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       const uint64_t t0 = globaltimer();
       auto drain = [&](uint64_t* bar, uint32_t parity) {
         while (!mbar_try_wait(bar, parity))
-          if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+          if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
       };
       if (qi > 0) drain(&sm.qd_full, (qi - 1) & 1);
       for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) drain(&full[u & 1], (u >> 1) & 1);
@@ -268,7 +268,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       mma_commit(&sm.mma_done);
       const uint64_t t0 = globaltimer();
       while (!mbar_try_wait(&sm.mma_done, 0))
-        if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+        if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
     }
   } else {
     const uint32_t quarter = warp & 3;
@@ -493,7 +493,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       const uint64_t t0 = globaltimer();
       auto drain = [&](uint64_t* bar, uint32_t parity) {
         while (!mbar_try_wait(bar, parity))
-          if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+          if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
       };
       if (ki > 0) drain(&sm.kv_full, (ki - 1) & 1);
       for (uint32_t u = (qd >= 2 ? qd - 2 : 0); u < qd; ++u) drain(&full[u & 1], (u >> 1) & 1);
@@ -579,7 +579,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       mma_commit(&sm.mma_done);
       const uint64_t t0 = globaltimer();
       while (!mbar_try_wait(&sm.mma_done, 0))
-        if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+        if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
     }
   } else {
     const uint32_t quarter = warp & 3;

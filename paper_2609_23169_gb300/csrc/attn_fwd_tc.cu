@@ -151,7 +151,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       const uint64_t t0 = globaltimer();
       auto drain = [&](uint64_t* bar, uint32_t parity) {
         while (!mbar_try_wait(bar, parity))
-          if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+          if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
       };
       if (qi > 0) drain(&sm.q_full, (qi - 1) & 1);
       for (uint32_t u = (kv >= kStages ? kv - kStages : 0); u < kv; ++u)
@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       mma_commit(&sm.mma_done);
       const uint64_t t0 = globaltimer();
       while (!mbar_try_wait(&sm.mma_done, 0))
-        if (globaltimer() - t0 > prm.timeout_ns) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+        if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
     }
   } else {
     // ------------------------------------------------------------- softmax

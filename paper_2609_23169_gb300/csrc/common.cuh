@@ -12,6 +12,11 @@
 
 namespace ut {
 
+// Limit for the drains on the way out of a kernel (its own in-flight TMA copies
+// and MMAs must land before the CTA frees TMEM and exits).  Independent of the
+// per-call wait limit, so that a tiny wait limit can never skip a drain.
+constexpr uint64_t kDrainTimeoutNs = 2000000000ull;
+
 // ------------------------------------------------------------------ status
 UT_DEV void set_status(int32_t* status, int32_t code) {
   if (status) atomicCAS(status, 0, code);
@@ -59,10 +64,16 @@ UT_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 
 // Bounded wait: returns false (and records UT_ERR_TIMEOUT, raises the CTA's
 // abort flag) if the phase with this parity has not completed within
-// timeout_ns, or if another role of the CTA has already aborted.
+// timeout_ns, or if another role of the CTA has already aborted.  A limit of 0
+// gives up at the first wait that is not already satisfied (diagnostics).
 UT_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int32_t* status,
                       uint64_t timeout_ns) {
   if (mbar_try_wait(bar, parity)) return true;
+  if (timeout_ns == 0) {
+    set_status(status, UT_ERR_TIMEOUT);
+    *abort_flag = 1;
+    return false;
+  }
   uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
