@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--sweep", action="store_true",
+                    help="2048-canvas sweep: one JSON line per (foreground, rho, block) point instead of the bench line")
     return ap.parse_args()
 
 
@@ -389,6 +391,75 @@ def oracle_sample(w, seconds: float):
     return flops / dt / 1e12, desc, dt
 
 
+def run_sweep(args):
+    """One line per point of the 2048-canvas sweep (foreground x rho x block):
+    device time of forward and backward, their TFLOP/s and % of the measured
+    peak, and the ratio to the same foreground's rho = 1 (dense-foreground)
+    point.  Not the benchmark line; the points are parity-test shapes."""
+    import torch
+    import __graft_entry__ as g
+    from paper_2609_23169_gb300 import path as P
+    from paper_2609_23169_gb300 import ultratex as u
+    from synth.workloads import SWEEP_BLOCK, SWEEP_FG, SWEEP_RHO, sweep2048
+
+    g.build()
+    dev = torch.device("cuda", 0)
+    peaks, src = load_peaks()
+    peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    steps = max(1, args.steps if args.steps != 10 else 2)
+    for fg in SWEEP_FG:
+        base = sweep2048(fg, 1.0, 128)
+        q, k, v, do = (x.to(dev) for x in (base.q(), base.k(), base.v(), base.dout()))
+        mask = torch.from_numpy(base.canvas_mask()).to(dev)
+        dense_ms = {}
+        for block in sorted(SWEEP_BLOCK, reverse=True):
+            for rho in sorted(SWEEP_RHO, reverse=True):
+                w = sweep2048(fg, rho, block)
+                line = {"sweep": True, "workload": w.name, "fg": fg, "rho": rho, "block": block, "N": w.N}
+                if block != 128:
+                    line["unavailable"] = "bf16 block size 64 has no tensor-core kernel yet (UT_ERR_UNSUPPORTED)"
+                    print(json.dumps(line), flush=True)
+                    continue
+                hp = P.HotPath(w.T, w.heads, w.head_dim, block, torch.bfloat16, u.UT_MASK_TOPK, rho=rho, device=dev)
+                N = hp.step(mask, q, k, v, do)
+                torch.cuda.synchronize()
+                nq = -(-N // block)
+                rp = hp.row_ptr[:w.heads * nq + 1].cpu().numpy()
+                ci = hp.col_idx[:int(rp[-1])].cpu().numpy()
+                f_fwd = retained_flops(rp, ci, N, block, w.head_dim)
+                ev = []
+                for _ in range(steps):
+                    Nn = hp.compact(mask, [q, k, v, do])
+                    hp.block_lists(Nn)
+                    a, b_, c_ = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+                    a.record()
+                    hp.forward(Nn)
+                    b_.record()
+                    hp.backward_pass(Nn)
+                    c_.record()
+                    hp.scatter(Nn)
+                    ev.append((a, b_, c_))
+                torch.cuda.synchronize()
+                u.check_status(hp.status)
+                fwd_ms = sum(a.elapsed_time(b_) for a, b_, _ in ev) / steps
+                bwd_ms = sum(b_.elapsed_time(c_) for _, b_, c_ in ev) / steps
+                if rho == 1.0:
+                    dense_ms[block] = (fwd_ms, bwd_ms)
+                d_f, d_b = dense_ms.get(block, (None, None))
+                line.update({"density": round(float(rp[-1]) / (w.heads * nq * nq), 4),
+                             "fwd_ms": round(fwd_ms, 3), "bwd_ms": round(bwd_ms, 3),
+                             "fwd_tflops": round(f_fwd / fwd_ms / 1e9, 1),
+                             "bwd_tflops": round(2.5 * f_fwd / bwd_ms / 1e9, 1),
+                             "fwd_pct_peak": round(100 * f_fwd / fwd_ms / 1e9 / peak, 1),
+                             "speedup_vs_dense_fg": {"fwd": round(d_f / fwd_ms, 2) if d_f else None,
+                                                     "bwd": round(d_b / bwd_ms, 2) if d_b else None},
+                             "peak": f"{peak} TFLOP/s ({src} bf16 burst)"})
+                print(json.dumps(line), flush=True)
+                del hp
+                torch.cuda.empty_cache()
+    return 0
+
+
 def cpu_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -402,6 +473,8 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     from synth import CONFIGS
+    if args.sweep:
+        return run_sweep(args)
     if args.impl == "reference":
         if rank != 0:
             return 0
