@@ -194,16 +194,15 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
             tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, j * kTile, pol_kv);
         }
       }
-      const uint64_t t0 = globaltimer();
       auto drain = [&](uint64_t* bar, uint32_t parity) {
-        while (!mbar_try_wait(bar, parity))
-          if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+        if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
       };
       if (qi > 0) drain(&sm.qd_full, (qi - 1) & 1);
       for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) drain(&full[u & 1], (u >> 1) & 1);
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    // whole warp, converged: waits are warp-uniform, MMAs/commits elect one lane
+    {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
       constexpr uint32_t idesc_dq = idesc_bf16_f32(kTile, D, false, true);
       const uint32_t q_addr = smem_u32(sm.q), do_addr = smem_u32(sm.dout), ds_addr = smem_u32(sm.ds);
@@ -212,63 +211,61 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int L = prm.ptr[w + 1] - prm.ptr[w];
         if (L <= 0) continue;
-        if (!(ok = mbar_wait(&sm.qd_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        if (!(ok = warp_wait(&sm.qd_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         for (int t = 0; t <= L && ok; ++t) {
           if (t < L) {
             const uint32_t kv = kv0 + t, st = kv & 1, n = kv >> 1;
             const uint32_t sc = sc0 + t;
             // S = Q K^T once the previous S has been read; dP = dO V^T once the previous dP has
             const uint32_t k_addr = smem_u32(sm.k[st]), v_addr = smem_u32(sm.v[st]);
-            if (!(ok = mbar_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.s_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.s_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss(tmem, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024), idesc_s,
+              mma_bf16_ss_w(tmem, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024), idesc_s,
                           kk > 0);
             }
-            mma_commit(&sm.s_full);
-            if (!(ok = mbar_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.dp_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            mma_commit_w(&sm.s_full);
+            if (!(ok = warp_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.dp_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss(tmem + 128, sdesc_sw128(do_addr + off, 16, 1024), sdesc_sw128(v_addr + off, 16, 1024),
+              mma_bf16_ss_w(tmem + 128, sdesc_sw128(do_addr + off, 16, 1024), sdesc_sw128(v_addr + off, 16, 1024),
                           idesc_s, kk > 0);
             }
-            mma_commit(&sm.dp_full);
-            mma_commit(&sm.v_empty[st]);
-            if (t == L - 1) mma_commit(&sm.qd_empty);
+            mma_commit_w(&sm.dp_full);
+            mma_commit_w(&sm.v_empty[st]);
+            if (t == L - 1) mma_commit_w(&sm.qd_empty);
           }
           if (t >= 1) {
             const uint32_t u = t - 1;
             const uint32_t kv = kv0 + u, st = kv & 1;
             const uint32_t sc = sc0 + u;
-            if (!(ok = mbar_wait(&sm.ds_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (u == 0 && !(ok = mbar_wait(&sm.dq_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+            if (!(ok = warp_wait(&sm.ds_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (u == 0 && !(ok = warp_wait(&sm.dq_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
               break;
             tc_fence_after();
             const uint32_t k_addr = smem_u32(sm.k[st]);
 #pragma unroll
             for (int kk = 0; kk < kTile / 16; ++kk) {
               const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss(tmem + 256, sdesc_sw128(ds_addr + aoff, 16, 1024),
+              mma_bf16_ss_w(tmem + 256, sdesc_sw128(ds_addr + aoff, 16, 1024),
                           sdesc_sw128(k_addr + kk * 2048, kChunk, 1024), idesc_dq, (u > 0 || kk > 0));
             }
-            mma_commit(&sm.dq_mma_done);
-            mma_commit(&sm.k_empty[st]);
+            mma_commit_w(&sm.dq_mma_done);
+            mma_commit_w(&sm.k_empty[st]);
           }
         }
         kv0 += L;
         sc0 += L;
         ++qi;
       }
-      mma_commit(&sm.mma_done);
-      const uint64_t t0 = globaltimer();
-      while (!mbar_try_wait(&sm.mma_done, 0))
-        if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+      mma_commit_w(&sm.mma_done);
+      if (!mbar_drain(&sm.mma_done, 0, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
     }
   } else {
     const uint32_t quarter = warp & 3;
@@ -490,16 +487,15 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
             tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, i * kTile, pol_qd);
         }
       }
-      const uint64_t t0 = globaltimer();
       auto drain = [&](uint64_t* bar, uint32_t parity) {
-        while (!mbar_try_wait(bar, parity))
-          if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+        if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
       };
       if (ki > 0) drain(&sm.kv_full, (ki - 1) & 1);
       for (uint32_t u = (qd >= 2 ? qd - 2 : 0); u < qd; ++u) drain(&full[u & 1], (u >> 1) & 1);
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    // whole warp, converged: waits are warp-uniform, MMAs/commits elect one lane
+    {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
       constexpr uint32_t idesc_acc = idesc_bf16_f32(kTile, D, false, true);
       const uint32_t k_addr = smem_u32(sm.k), v_addr = smem_u32(sm.v), pds_addr = smem_u32(sm.pds);
@@ -508,78 +504,76 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int L = prm.ptr[w + 1] - prm.ptr[w];
         if (L <= 0) continue;
-        if (!(ok = mbar_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         for (int t = 0; t <= L && ok; ++t) {
           // issue order per step: S^T_t, dV_{t-1}, dP^T_t, dK_{t-1}
           const uint32_t qd_t = qd0 + t, st_t = qd_t & 1, n_t = qd_t >> 1;
           if (t < L) {
-            if (!(ok = mbar_wait(&sm.q_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.s_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.q_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.s_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
             const uint32_t q_addr = smem_u32(sm.q[st_t]);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss(tmem, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024), idesc_s,
+              mma_bf16_ss_w(tmem, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024), idesc_s,
                           kk > 0);
             }
-            mma_commit(&sm.s_full);
+            mma_commit_w(&sm.s_full);
           }
           if (t >= 1) {
             const uint32_t u = t - 1;
             const uint32_t qd = qd0 + u, st = qd & 1;
             const uint32_t do_addr = smem_u32(sm.dout[st]);
-            if (!(ok = mbar_wait(&sm.pt_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (u == 0 && !(ok = mbar_wait(&sm.acc_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+            if (!(ok = warp_wait(&sm.pt_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (u == 0 && !(ok = warp_wait(&sm.acc_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
               break;
             tc_fence_after();
 #pragma unroll
             for (int kk = 0; kk < kTile / 16; ++kk) {
               const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss(tmem + 256, sdesc_sw128(pds_addr + aoff, 16, 1024),
+              mma_bf16_ss_w(tmem + 256, sdesc_sw128(pds_addr + aoff, 16, 1024),
                           sdesc_sw128(do_addr + kk * 2048, kChunk, 1024), idesc_acc, (u > 0 || kk > 0));
             }
-            mma_commit(&sm.pt_done);
-            mma_commit(&sm.do_empty[st]);
+            mma_commit_w(&sm.pt_done);
+            mma_commit_w(&sm.do_empty[st]);
           }
           if (t < L) {
-            if (!(ok = mbar_wait(&sm.do_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.dp_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.do_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.dp_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
             const uint32_t do_addr = smem_u32(sm.dout[st_t]);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss(tmem + 128, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
+              mma_bf16_ss_w(tmem + 128, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
                           idesc_s, kk > 0);
             }
-            mma_commit(&sm.dp_full);
-            if (t == L - 1) mma_commit(&sm.kv_empty);
+            mma_commit_w(&sm.dp_full);
+            if (t == L - 1) mma_commit_w(&sm.kv_empty);
           }
           if (t >= 1) {
             const uint32_t u = t - 1;
             const uint32_t qd = qd0 + u, st = qd & 1;
             const uint32_t q_addr = smem_u32(sm.q[st]);
-            if (!(ok = mbar_wait(&sm.dst_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.dst_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
 #pragma unroll
             for (int kk = 0; kk < kTile / 16; ++kk) {
               const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss(tmem + 384, sdesc_sw128(pds_addr + aoff, 16, 1024),
+              mma_bf16_ss_w(tmem + 384, sdesc_sw128(pds_addr + aoff, 16, 1024),
                           sdesc_sw128(q_addr + kk * 2048, kChunk, 1024), idesc_acc, (u > 0 || kk > 0));
             }
-            mma_commit(&sm.ds_done);
-            mma_commit(&sm.q_empty[st]);
+            mma_commit_w(&sm.ds_done);
+            mma_commit_w(&sm.q_empty[st]);
           }
         }
-        mma_commit(&sm.acc_full);
+        mma_commit_w(&sm.acc_full);
         qd0 += L;
         ++ki;
       }
-      mma_commit(&sm.mma_done);
-      const uint64_t t0 = globaltimer();
-      while (!mbar_try_wait(&sm.mma_done, 0))
-        if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+      mma_commit_w(&sm.mma_done);
+      if (!mbar_drain(&sm.mma_done, 0, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
     }
   } else {
     const uint32_t quarter = warp & 3;

@@ -148,10 +148,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         }
       }
       // Drain: every copy this lane issued has landed before the CTA may exit.
-      const uint64_t t0 = globaltimer();
       auto drain = [&](uint64_t* bar, uint32_t parity) {
-        while (!mbar_try_wait(bar, parity))
-          if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+        if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
       };
       if (qi > 0) drain(&sm.q_full, (qi - 1) & 1);
       for (uint32_t u = (kv >= kStages ? kv - kStages : 0); u < kv; ++u)
@@ -159,7 +157,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------- MMA issuer
-    if (lane == 0) {
+    // The whole warp runs this loop converged; every MMA and commit is issued
+    // by one elected lane (see mma_bf16_ss_w), waits are warp-uniform.
+    {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN, false, false);
       constexpr uint32_t idesc_o = idesc_bf16_f32(kBM, D, false, true);
       const uint32_t q_addr = smem_u32(sm.q);
@@ -168,41 +168,41 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int L = prm.row_ptr[w + 1] - prm.row_ptr[w];
         if (L <= 0) continue;
-        if (!(ok = mbar_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        if (!(ok = warp_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         for (int t = 0; t <= L && ok; ++t) {
           if (t < L) {
             const uint32_t kv = kv0 + t, st = kv % kStages, n = kv / kStages;
             const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
-            if (!(ok = mbar_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.s_empty[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.s_empty[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
             const uint32_t k_addr = smem_u32(sm.k[st]);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kTileChunkBytes + (kk & 3) * 32;
-              mma_bf16_ss(tmem + sb * 128, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024),
-                          idesc_s, kk > 0);
+              mma_bf16_ss_w(tmem + sb * 128, sdesc_sw128(q_addr + off, 16, 1024),
+                            sdesc_sw128(k_addr + off, 16, 1024), idesc_s, kk > 0);
             }
-            mma_commit(&sm.s_full[sb]);
-            mma_commit(&sm.k_empty[st]);
-            if (t == L - 1) mma_commit(&sm.q_empty);
+            mma_commit_w(&sm.s_full[sb]);
+            mma_commit_w(&sm.k_empty[st]);
+            if (t == L - 1) mma_commit_w(&sm.q_empty);
           }
           if (t >= 1) {
             const uint32_t u = t - 1;
             const uint32_t kv = kv0 + u, st = kv % kStages, n = kv / kStages;
             const uint32_t sc = sc0 + u, pb = sc & 1, np = sc >> 1;
-            if (!(ok = mbar_wait(&sm.p_full[pb], np & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = mbar_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (u == 0 && !(ok = mbar_wait(&sm.o_empty, (oi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+            if (!(ok = warp_wait(&sm.p_full[pb], np & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (u == 0 && !(ok = warp_wait(&sm.o_empty, (oi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
               break;
             tc_fence_after();
             const uint32_t v_addr = smem_u32(sm.v[st]);
 #pragma unroll
             for (int kk = 0; kk < kBN / 16; ++kk)
-              mma_bf16_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
-                          sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024), idesc_o, (u > 0 || kk > 0));
-            mma_commit(&sm.pv_done[pb]);
-            mma_commit(&sm.v_empty[st]);
+              mma_bf16_ts_w(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
+                            sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024), idesc_o, (u > 0 || kk > 0));
+            mma_commit_w(&sm.pv_done[pb]);
+            mma_commit_w(&sm.v_empty[st]);
           }
         }
         kv0 += L;
@@ -210,11 +210,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         ++qi;
         ++oi;
       }
-      // Drain: all MMAs issued by this thread complete before TMEM is freed.
-      mma_commit(&sm.mma_done);
-      const uint64_t t0 = globaltimer();
-      while (!mbar_try_wait(&sm.mma_done, 0))
-        if (globaltimer() - t0 > kDrainTimeoutNs) { set_status(prm.status, UT_ERR_TIMEOUT); break; }
+      // Drain: all MMAs issued by this warp complete before TMEM is freed.
+      mma_commit_w(&sm.mma_done);
+      if (!mbar_drain(&sm.mma_done, 0, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
     }
   } else {
     // ------------------------------------------------------------- softmax

@@ -66,26 +66,76 @@ UT_DEV bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // abort flag) if the phase with this parity has not completed within
 // timeout_ns, or if another role of the CTA has already aborted.  A limit of 0
 // gives up at the first wait that is not already satisfied (diagnostics).
+// The spin loop lives inside one asm block: a loop written in C++ around the
+// wait, placed between tcgen05.mma groups, keeps the tensor pipe from
+// streaming consecutive MMAs (measured: ~2x fewer MMAs per cycle).
 UT_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int32_t* status,
                       uint64_t timeout_ns) {
-  if (mbar_try_wait(bar, parity)) return true;
-  if (timeout_ns == 0) {
+  uint32_t r;  // 1 = phase complete, 0 = timed out, 2 = CTA already aborted
+  asm volatile(
+      "{\n\t"
+      ".reg .pred p, q;\n\t"
+      ".reg .u64 t0, t1;\n\t"
+      ".reg .u32 ab;\n\t"
+      "mov.u32 %0, 1;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "@p bra UT_WAIT_DONE;\n\t"
+      "setp.eq.u64 q, %4, 0;\n\t"
+      "@q bra UT_WAIT_TIMEOUT;\n\t"
+      "mov.u64 t0, %%globaltimer;\n\t"
+      "UT_WAIT_LOOP:\n\t"
+      "ld.volatile.shared.u32 ab, [%3];\n\t"
+      "setp.ne.u32 q, ab, 0;\n\t"
+      "@q bra UT_WAIT_ABORT;\n\t"
+      "mov.u64 t1, %%globaltimer;\n\t"
+      "sub.u64 t1, t1, t0;\n\t"
+      "setp.gt.u64 q, t1, %4;\n\t"
+      "@q bra UT_WAIT_TIMEOUT;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "@!p bra UT_WAIT_LOOP;\n\t"
+      "bra UT_WAIT_DONE;\n\t"
+      "UT_WAIT_ABORT:\n\t"
+      "mov.u32 %0, 2;\n\t"
+      "bra UT_WAIT_DONE;\n\t"
+      "UT_WAIT_TIMEOUT:\n\t"
+      "mov.u32 %0, 0;\n\t"
+      "UT_WAIT_DONE:\n\t"
+      "}"
+      : "=r"(r)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(smem_u32(const_cast<int*>(abort_flag))), "l"(timeout_ns)
+      : "memory");
+  if (r == 1) return true;
+  if (r == 0) {
     set_status(status, UT_ERR_TIMEOUT);
     *abort_flag = 1;
-    return false;
   }
-  uint64_t t0 = globaltimer();
-  for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63) == 0) {
-      if (*abort_flag) return false;
-      if (globaltimer() - t0 > timeout_ns) {
-        set_status(status, UT_ERR_TIMEOUT);
-        *abort_flag = 1;
-        return false;
-      }
-    }
-  }
+  return false;
+}
+
+// Unbounded-count but time-bounded drain wait (no abort check): used on the way
+// out of a kernel for the CTA's own copies and MMAs.
+UT_DEV bool mbar_drain(uint64_t* bar, uint32_t parity, uint64_t timeout_ns) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t"
+      ".reg .pred p, q;\n\t"
+      ".reg .u64 t0, t1;\n\t"
+      "mov.u32 %0, 1;\n\t"
+      "mov.u64 t0, %%globaltimer;\n\t"
+      "UT_DRAIN_LOOP:\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "@p bra UT_DRAIN_DONE;\n\t"
+      "mov.u64 t1, %%globaltimer;\n\t"
+      "sub.u64 t1, t1, t0;\n\t"
+      "setp.gt.u64 q, t1, %3;\n\t"
+      "@!q bra UT_DRAIN_LOOP;\n\t"
+      "mov.u32 %0, 0;\n\t"
+      "UT_DRAIN_DONE:\n\t"
+      "}"
+      : "=r"(r)
+      : "r"(smem_u32(bar)), "r"(parity), "l"(timeout_ns)
+      : "memory");
+  return r == 1;
 }
 
 // Warp-collective form: every lane waits, and the warp agrees on the outcome
@@ -160,6 +210,36 @@ UT_DEV void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32
       "setp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
       "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Warp-collective forms: the whole (converged) warp executes them and the
+// instruction is issued by one elected lane (always the same lane while the
+// warp is fully active, so commits track that lane's MMAs).
+UT_DEV void mma_bf16_ss_w(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred e, p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+UT_DEV void mma_bf16_ts_w(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred e, p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+UT_DEV void mma_commit_w(uint64_t* bar) {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(
+          smem_u32(bar))
       : "memory");
 }
 
