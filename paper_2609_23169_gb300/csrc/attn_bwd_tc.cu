@@ -27,7 +27,8 @@
 namespace ut {
 
 constexpr int kTile = 128;
-constexpr int kBwdThreads = 192;
+constexpr int kDqThreads = 320;    // dQ kernel: 2 role warps + 8 elementwise
+constexpr int kDkdvThreads = 320;  // dK/dV kernel: 2 role warps + 8 elementwise
 constexpr uint32_t kChunk = 128 * 128;  // one 128-row x 128-byte swizzled sub-tile
 
 // ------------------------------------------------------------- preprocess
@@ -84,17 +85,21 @@ struct BwdParams {
 // =========================================================================
 //                                  dQ
 // =========================================================================
+// dQ kernel rings: K is held from S = Q K^T until dQ += dS K, so it gets the
+// deeper ring; V is released right after dP = dO V^T.  dS lives in TMEM.
+constexpr int kDqKStages = 3, kDqVStages = 2;
+constexpr uint32_t kDqColDs = 384;  // TMEM columns of dS (bf16 pairs): [384, 448)
+
 template <int D>
 struct DqSmem {
   static constexpr int kC = D / 64;
   static constexpr uint32_t kTileBytes = kTile * D * 2;
   alignas(1024) uint8_t q[kTileBytes];
   alignas(1024) uint8_t dout[kTileBytes];
-  alignas(1024) uint8_t k[2][kTileBytes];
-  alignas(1024) uint8_t v[2][kTileBytes];
-  alignas(1024) uint8_t ds[kTile * kTile * 2];
+  alignas(1024) uint8_t k[kDqKStages][kTileBytes];
+  alignas(1024) uint8_t v[kDqVStages][kTileBytes];
   uint64_t qd_full, qd_empty;
-  uint64_t k_full[2], v_full[2], k_empty[2], v_empty[2];
+  uint64_t k_full[kDqKStages], k_empty[kDqKStages], v_full[kDqVStages], v_empty[kDqVStages];
   uint64_t s_full, s_empty, dp_full, dp_empty, ds_full, dq_mma_done, dq_empty, mma_done;
   uint32_t tmem_base;
   int abort_flag;
@@ -108,7 +113,7 @@ UT_DEV void tmem_ld64(uint32_t taddr, uint32_t* r) {
 }
 
 template <int D>
-__global__ void __launch_bounds__(kBwdThreads, 1)
+__global__ void __launch_bounds__(kDqThreads, 1)
     bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
                   const BwdParams prm) {
@@ -125,19 +130,21 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(&sm.qd_full, 1);
     mbar_init(&sm.qd_empty, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kDqKStages; ++s) {
       mbar_init(&sm.k_full[s], 1);
-      mbar_init(&sm.v_full[s], 1);
       mbar_init(&sm.k_empty[s], 1);
+    }
+    for (int s = 0; s < kDqVStages; ++s) {
+      mbar_init(&sm.v_full[s], 1);
       mbar_init(&sm.v_empty[s], 1);
     }
     mbar_init(&sm.s_full, 1);
-    mbar_init(&sm.s_empty, 4);
+    mbar_init(&sm.s_empty, 8);
     mbar_init(&sm.dp_full, 1);
-    mbar_init(&sm.dp_empty, 4);
-    mbar_init(&sm.ds_full, 4);
+    mbar_init(&sm.dp_empty, 8);
+    mbar_init(&sm.ds_full, 8);
     mbar_init(&sm.dq_mma_done, 1);
-    mbar_init(&sm.dq_empty, 4);
+    mbar_init(&sm.dq_empty, 8);
     mbar_init(&sm.mma_done, 1);
     sm.abort_flag = 0;
     fence_barrier_init();
@@ -169,6 +176,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       uint64_t* empty = is_k ? sm.k_empty : sm.v_empty;
       uint8_t* ring = is_k ? &sm.k[0][0] : &sm.v[0][0];
       const void* tmap = is_k ? static_cast<const void*>(&tm_k) : static_cast<const void*>(&tm_v);
+      const uint32_t nst = is_k ? kDqKStages : kDqVStages;
       uint32_t qi = 0, kv = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
@@ -186,8 +194,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         }
         for (int t = 0; t < L; ++t, ++kv) {
           const int j = prm.idx[beg + t];
-          const int st = kv & 1;
-          const uint32_t n = kv >> 1;
+          const uint32_t st = kv % nst, n = kv / nst;
           if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
           mbar_expect_tx(&full[st], TB);
           for (int c = 0; c < C; ++c)
@@ -198,14 +205,14 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
       };
       if (qi > 0) drain(&sm.qd_full, (qi - 1) & 1);
-      for (uint32_t u = (kv >= 2 ? kv - 2 : 0); u < kv; ++u) drain(&full[u & 1], (u >> 1) & 1);
+      for (uint32_t u = (kv >= nst ? kv - nst : 0); u < kv; ++u) drain(&full[u % nst], (u / nst) & 1);
     }
   } else if (warp == 1) {
     // whole warp, converged: waits are warp-uniform, MMAs/commits elect one lane
     {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
       constexpr uint32_t idesc_dq = idesc_bf16_f32(kTile, D, false, true);
-      const uint32_t q_addr = smem_u32(sm.q), do_addr = smem_u32(sm.dout), ds_addr = smem_u32(sm.ds);
+      const uint32_t q_addr = smem_u32(sm.q), do_addr = smem_u32(sm.dout);
       uint32_t qi = 0, kv0 = 0, sc0 = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
@@ -214,11 +221,12 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         if (!(ok = warp_wait(&sm.qd_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         for (int t = 0; t <= L && ok; ++t) {
           if (t < L) {
-            const uint32_t kv = kv0 + t, st = kv & 1, n = kv >> 1;
+            const uint32_t kv = kv0 + t, sk = kv % kDqKStages, nk = kv / kDqKStages;
+            const uint32_t sv = kv % kDqVStages, nv = kv / kDqVStages;
             const uint32_t sc = sc0 + t;
             // S = Q K^T once the previous S has been read; dP = dO V^T once the previous dP has
-            const uint32_t k_addr = smem_u32(sm.k[st]), v_addr = smem_u32(sm.v[st]);
-            if (!(ok = warp_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            const uint32_t k_addr = smem_u32(sm.k[sk]), v_addr = smem_u32(sm.v[sv]);
+            if (!(ok = warp_wait(&sm.k_full[sk], nk & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             if (!(ok = warp_wait(&sm.s_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
 #pragma unroll
@@ -228,7 +236,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
                           kk > 0);
             }
             mma_commit_w(&sm.s_full);
-            if (!(ok = warp_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.v_full[sv], nv & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             if (!(ok = warp_wait(&sm.dp_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
 #pragma unroll
@@ -238,26 +246,24 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
                           idesc_s, kk > 0);
             }
             mma_commit_w(&sm.dp_full);
-            mma_commit_w(&sm.v_empty[st]);
+            mma_commit_w(&sm.v_empty[sv]);
             if (t == L - 1) mma_commit_w(&sm.qd_empty);
           }
           if (t >= 1) {
             const uint32_t u = t - 1;
-            const uint32_t kv = kv0 + u, st = kv & 1;
+            const uint32_t kv = kv0 + u, sk = kv % kDqKStages;
             const uint32_t sc = sc0 + u;
             if (!(ok = warp_wait(&sm.ds_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
             if (u == 0 && !(ok = warp_wait(&sm.dq_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
               break;
             tc_fence_after();
-            const uint32_t k_addr = smem_u32(sm.k[st]);
+            const uint32_t k_addr = smem_u32(sm.k[sk]);
 #pragma unroll
-            for (int kk = 0; kk < kTile / 16; ++kk) {
-              const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem + 256, sdesc_sw128(ds_addr + aoff, 16, 1024),
-                          sdesc_sw128(k_addr + kk * 2048, kChunk, 1024), idesc_dq, (u > 0 || kk > 0));
-            }
+            for (int kk = 0; kk < kTile / 16; ++kk)
+              mma_bf16_ts_w(tmem + 256, tmem + kDqColDs + kk * 8, sdesc_sw128(k_addr + kk * 2048, kChunk, 1024),
+                            idesc_dq, (u > 0 || kk > 0));
             mma_commit_w(&sm.dq_mma_done);
-            mma_commit_w(&sm.k_empty[st]);
+            mma_commit_w(&sm.k_empty[sk]);
           }
         }
         kv0 += L;
@@ -268,9 +274,15 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       if (!mbar_drain(&sm.mma_done, 0, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
     }
   } else {
+    // 8 elementwise warps: warps w and w+4 share TMEM lane quarter (w & 3),
+    // i.e. the same 32 query rows, and split the 128 key columns (and the D
+    // output columns) into halves; a half is one 128-byte swizzle chunk of dS.
     const uint32_t quarter = warp & 3;
+    const uint32_t half = (warp - 2) >> 2;
     const uint32_t row = quarter * 32 + lane;
     const uint32_t lane_base = (quarter * 32) << 16;
+    constexpr int HC = kTile / 2;
+    constexpr int HD = D / 2;
     const float c = prm.scale_log2;
     uint32_t sc0 = 0;
     bool ok = true;
@@ -279,10 +291,10 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
       const int64_t grow = (int64_t)i * kTile + row;
       const bool row_ok = grow < prm.N;
-      __nv_bfloat16* orow = prm.out0 + grow * prm.rs + (int64_t)h * D;
+      __nv_bfloat16* orow = prm.out0 + grow * prm.rs + (int64_t)h * D + half * HD;
       if (L <= 0) {
         if (row_ok)
-          for (int e = 0; e < D; e += 8) *reinterpret_cast<uint4*>(orow + e) = make_uint4(0, 0, 0, 0);
+          for (int e = 0; e < HD; e += 8) *reinterpret_cast<uint4*>(orow + e) = make_uint4(0, 0, 0, 0);
         continue;
       }
       const float lse2 = prm.lse2[(int64_t)h * prm.Np + grow];
@@ -292,62 +304,55 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         const uint32_t sc = sc0 + t;
         const int j = j_cur;
         if (t + 1 < L) j_cur = prm.idx[beg + t + 1];  // prefetch the next key block index
-        const int64_t nv = prm.N - (int64_t)j * kTile;
+        const int64_t nv = prm.N - (int64_t)j * kTile - (int64_t)half * HC;  // valid columns of this half
         if (!(ok = warp_wait(&sm.s_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
-        float p[kTile];
+        float p[HC];
         {
-          uint32_t r[kTile];
-#pragma unroll
-          for (int g = 0; g < kTile / 32; ++g)
-            tmem_ld32(tmem + lane_base + g * 32, *reinterpret_cast<uint32_t(*)[32]>(&r[g * 32]));
-          tmem_wait_ld();
+          uint32_t r[HC];
+          tmem_ld64(tmem + lane_base + half * HC, r);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.s_empty);
 #pragma unroll
-          for (int col = 0; col < kTile; ++col)
-            p[col] = col < nv ? ex2_approx(fmaf(__uint_as_float(r[col]), c, -lse2)) : 0.f;
+          for (int x = 0; x < HC; ++x) p[x] = ex2_approx(fmaf(__uint_as_float(r[x]), c, -lse2));
+          if (nv < HC) {  // ragged last key block: columns past N do not exist
+#pragma unroll
+            for (int x = 0; x < HC; ++x)
+              if (x >= nv) p[x] = 0.f;
+          }
         }
         if (!(ok = warp_wait(&sm.dp_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
         // dS buffer is free once the previous tile's dQ MMA finished
         if (!(ok = warp_wait(&sm.dq_mma_done, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        const uint32_t ds_row = smem_u32(sm.ds) + row * 128;
+        tc_fence_after();
+        {
+          uint32_t r[HC];
+          tmem_ld64(tmem + lane_base + 128 + half * HC, r);
+          uint32_t pk[HC / 2];
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          uint32_t r[64];
-          tmem_ld64(tmem + lane_base + 128 + half * 64, r);
-          if (half == 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.dp_empty);
-          }
-#pragma unroll
-          for (int u8 = 0; u8 < 8; ++u8) {
-            const int col = half * 64 + u8 * 8;
-            uint32_t pk[4];
-#pragma unroll
-            for (int x = 0; x < 8; x += 2)
-              pk[x / 2] = pack_bf16x2(p[col + x] * (__uint_as_float(r[u8 * 8 + x]) - Dr),
-                                      p[col + x + 1] * (__uint_as_float(r[u8 * 8 + x + 1]) - Dr));
-            const uint32_t u = half * 8 + u8;  // 16-byte unit (8 keys) within the 128-key row
-            const uint32_t chunk = u >> 3, unit = u & 7;
-            st_shared_v4(ds_row + chunk * kChunk + ((unit ^ (row & 7)) << 4), pk[0], pk[1], pk[2], pk[3]);
-          }
+          for (int x = 0; x < HC; x += 2)
+            pk[x / 2] = pack_bf16x2(p[x] * (__uint_as_float(r[x]) - Dr), p[x + 1] * (__uint_as_float(r[x + 1]) - Dr));
+          // dS (bf16 pairs) into TMEM: this half's 64 keys are columns [kDqColDs + 32*half, +32)
+          tmem_st32(tmem + lane_base + kDqColDs + half * (HC / 2), pk);
+          tmem_wait_st();
         }
-        fence_proxy_async_smem();
+        tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.ds_full);
+        if (lane == 0) {
+          mbar_arrive(&sm.dp_empty);
+          mbar_arrive(&sm.ds_full);
+        }
       }
       if (!ok) break;
       const uint32_t last = sc0 + L - 1;
       if (!(ok = warp_wait(&sm.dq_mma_done, last & 1, abort_flag, prm.status, prm.timeout_ns))) break;
       tc_fence_after();
 #pragma unroll
-      for (int g = 0; g < D / 32; ++g) {
+      for (int g = 0; g < HD / 32; ++g) {
         uint32_t r[32];
-        tmem_ld32(tmem + lane_base + 256 + g * 32, r);
+        tmem_ld32(tmem + lane_base + 256 + half * HD + g * 32, r);
         tmem_wait_ld();
         if (row_ok) {
 #pragma unroll
@@ -396,7 +401,7 @@ struct DkdvSmem {
 };
 
 template <int D>
-__global__ void __launch_bounds__(kBwdThreads, 1)
+__global__ void __launch_bounds__(kDkdvThreads, 1)
     bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
                     const BwdParams prm) {
@@ -420,18 +425,18 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       mbar_init(&sm.do_empty[s], 1);
     }
     mbar_init(&sm.s_full, 1);
-    mbar_init(&sm.s_empty, 4);
+    mbar_init(&sm.s_empty, 8);
     mbar_init(&sm.dp_full, 1);
-    mbar_init(&sm.dp_empty, 4);
-    mbar_init(&sm.pt_full, 4);
+    mbar_init(&sm.dp_empty, 8);
+    mbar_init(&sm.pt_full, 8);
     mbar_init(&sm.pt_done, 1);
-    mbar_init(&sm.dst_full, 4);
+    mbar_init(&sm.dst_full, 8);
     mbar_init(&sm.ds_done, 1);
     mbar_init(&sm.acc_full, 1);
-    mbar_init(&sm.acc_empty, 4);
+    mbar_init(&sm.acc_empty, 8);
     mbar_init(&sm.mma_done, 1);
-    mbar_init(&sm.rowvec_full[0], 128);
-    mbar_init(&sm.rowvec_full[1], 128);
+    mbar_init(&sm.rowvec_full[0], 256);
+    mbar_init(&sm.rowvec_full[1], 256);
     sm.abort_flag = 0;
     fence_barrier_init();
   }
@@ -506,21 +511,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         if (L <= 0) continue;
         if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         for (int t = 0; t <= L && ok; ++t) {
-          // issue order per step: S^T_t, dV_{t-1}, dP^T_t, dK_{t-1}
+          // issue order per step: dV_{t-1}, S^T_t, dP^T_t, dK_{t-1} (dV first: it only
+          // needs P^T_{t-1}, so it never waits behind the Q ring)
           const uint32_t qd_t = qd0 + t, st_t = qd_t & 1, n_t = qd_t >> 1;
-          if (t < L) {
-            if (!(ok = warp_wait(&sm.q_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = warp_wait(&sm.s_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            tc_fence_after();
-            const uint32_t q_addr = smem_u32(sm.q[st_t]);
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024), idesc_s,
-                          kk > 0);
-            }
-            mma_commit_w(&sm.s_full);
-          }
           if (t >= 1) {
             const uint32_t u = t - 1;
             const uint32_t qd = qd0 + u, st = qd & 1;
@@ -537,6 +530,19 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
             }
             mma_commit_w(&sm.pt_done);
             mma_commit_w(&sm.do_empty[st]);
+          }
+          if (t < L) {
+            if (!(ok = warp_wait(&sm.q_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.s_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+            const uint32_t q_addr = smem_u32(sm.q[st_t]);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss_w(tmem, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024), idesc_s,
+                          kk > 0);
+            }
+            mma_commit_w(&sm.s_full);
           }
           if (t < L) {
             if (!(ok = warp_wait(&sm.do_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -576,10 +582,17 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       if (!mbar_drain(&sm.mma_done, 0, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
     }
   } else {
+    // 8 elementwise warps: warps w and w+4 share TMEM lane quarter (w & 3),
+    // i.e. the same 32 key rows, and split the 128 query columns (and the D
+    // output columns) into halves.  A half is exactly one 128-byte swizzle
+    // chunk of the shared P^T / dS^T tile.
     const uint32_t quarter = warp & 3;
+    const uint32_t half = (warp - 2) >> 2;
     const uint32_t krow = quarter * 32 + lane;          // key row of the tile = TMEM lane
-    const uint32_t tid = threadIdx.x - 64;               // 0..127 within the elementwise group
+    const uint32_t tid = threadIdx.x - 64;               // 0..255 within the elementwise group
     const uint32_t lane_base = (quarter * 32) << 16;
+    constexpr int HC = kTile / 2;                        // query columns per half
+    constexpr int HD = D / 2;                            // output columns per half
     const float c = prm.scale_log2;
     uint32_t qd0 = 0, ki = 0;
     bool ok = true;
@@ -588,43 +601,41 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
       const int64_t gk = (int64_t)j * kTile + krow;
       const bool row_ok = gk < prm.N;
-      __nv_bfloat16* dv_row = prm.out0 + gk * prm.rs + (int64_t)h * D;
-      __nv_bfloat16* dk_row = prm.out1 + gk * prm.rs + (int64_t)h * D;
+      __nv_bfloat16* dv_row = prm.out0 + gk * prm.rs + (int64_t)h * D + half * HD;
+      __nv_bfloat16* dk_row = prm.out1 + gk * prm.rs + (int64_t)h * D + half * HD;
       if (L <= 0) {
         if (row_ok)
-          for (int e = 0; e < D; e += 8) {
+          for (int e = 0; e < HD; e += 8) {
             *reinterpret_cast<uint4*>(dv_row + e) = make_uint4(0, 0, 0, 0);
             *reinterpret_cast<uint4*>(dk_row + e) = make_uint4(0, 0, 0, 0);
           }
         continue;
       }
+      const uint32_t pds_chunk = smem_u32(sm.pds) + half * kChunk + krow * 128;
       for (int t = 0; t < L; ++t) {
         const uint32_t qd = qd0 + t;
         const int i = prm.idx[beg + t];
         // this pair's query-row LSE*log2e and D into the shared double buffer
         // (buffer qd&1 was last read in pair qd-2, which every thread finished
         //  before arriving for pair qd-1)
-        sm.lse2[qd & 1][tid] = prm.lse2[(int64_t)h * prm.Np + (int64_t)i * kTile + tid];
-        sm.dsum[qd & 1][tid] = prm.dsum[(int64_t)h * prm.Np + (int64_t)i * kTile + tid];
+        if (tid < kTile) sm.lse2[qd & 1][tid] = prm.lse2[(int64_t)h * prm.Np + (int64_t)i * kTile + tid];
+        else sm.dsum[qd & 1][tid - kTile] = prm.dsum[(int64_t)h * prm.Np + (int64_t)i * kTile + tid - kTile];
         mbar_arrive(&sm.rowvec_full[qd & 1]);
         if (!(ok = warp_wait(&sm.rowvec_full[qd & 1], (qd >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
           break;
-        const float* ls = sm.lse2[qd & 1];
-        const float* ds_v = sm.dsum[qd & 1];
+        const float* ls = sm.lse2[qd & 1] + half * HC;
+        const float* ds_v = sm.dsum[qd & 1] + half * HC;
         if (!(ok = warp_wait(&sm.s_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
-        float p[kTile];
+        float p[HC];
         {
-          uint32_t r[kTile];
-#pragma unroll
-          for (int g = 0; g < kTile / 32; ++g)
-            tmem_ld32(tmem + lane_base + g * 32, *reinterpret_cast<uint32_t(*)[32]>(&r[g * 32]));
-          tmem_wait_ld();
+          uint32_t r[HC];
+          tmem_ld64(tmem + lane_base + half * HC, r);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.s_empty);
 #pragma unroll
-          for (int x = 0; x < kTile; x += 4) {
+          for (int x = 0; x < HC; x += 4) {
             const float4 l4 = *reinterpret_cast<const float4*>(ls + x);
             p[x + 0] = ex2_approx(fmaf(__uint_as_float(r[x + 0]), c, -l4.x));
             p[x + 1] = ex2_approx(fmaf(__uint_as_float(r[x + 1]), c, -l4.y));
@@ -634,47 +645,37 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         }
         // the shared P/dS tile is free once the previous pair's dK MMA finished
         if (!(ok = warp_wait(&sm.ds_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        const uint32_t pds_row = smem_u32(sm.pds) + krow * 128;
 #pragma unroll
-        for (int u = 0; u < kTile / 8; ++u) {
-          const uint32_t chunk = u >> 3, unit = u & 7;
-          st_shared_v4(pds_row + chunk * kChunk + ((unit ^ (krow & 7)) << 4), pack_bf16x2(p[8 * u], p[8 * u + 1]),
+        for (int u = 0; u < HC / 8; ++u)
+          st_shared_v4(pds_chunk + ((u ^ (krow & 7)) << 4), pack_bf16x2(p[8 * u], p[8 * u + 1]),
                        pack_bf16x2(p[8 * u + 2], p[8 * u + 3]), pack_bf16x2(p[8 * u + 4], p[8 * u + 5]),
                        pack_bf16x2(p[8 * u + 6], p[8 * u + 7]));
-        }
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.pt_full);
-        uint32_t dsk[kTile / 2];
+        uint32_t dsk[HC / 2];
         if (!(ok = warp_wait(&sm.dp_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
+        {
+          uint32_t r[HC];
+          tmem_ld64(tmem + lane_base + 128 + half * HC, r);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.dp_empty);
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          uint32_t r[64];
-          tmem_ld64(tmem + lane_base + 128 + half * 64, r);
-          if (half == 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&sm.dp_empty);
-          }
-#pragma unroll
-          for (int x = 0; x < 64; x += 4) {
-            const int col = half * 64 + x;
-            const float4 d4 = *reinterpret_cast<const float4*>(ds_v + col);
-            dsk[col / 2] = pack_bf16x2(p[col] * (__uint_as_float(r[x]) - d4.x),
-                                       p[col + 1] * (__uint_as_float(r[x + 1]) - d4.y));
-            dsk[col / 2 + 1] = pack_bf16x2(p[col + 2] * (__uint_as_float(r[x + 2]) - d4.z),
-                                           p[col + 3] * (__uint_as_float(r[x + 3]) - d4.w));
+          for (int x = 0; x < HC; x += 4) {
+            const float4 d4 = *reinterpret_cast<const float4*>(ds_v + x);
+            dsk[x / 2] = pack_bf16x2(p[x] * (__uint_as_float(r[x]) - d4.x), p[x + 1] * (__uint_as_float(r[x + 1]) - d4.y));
+            dsk[x / 2 + 1] =
+                pack_bf16x2(p[x + 2] * (__uint_as_float(r[x + 2]) - d4.z), p[x + 3] * (__uint_as_float(r[x + 3]) - d4.w));
           }
         }
         // overwrite P^T with dS^T once the dV MMA has read P^T
         if (!(ok = warp_wait(&sm.pt_done, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
 #pragma unroll
-        for (int u = 0; u < kTile / 8; ++u) {
-          const uint32_t chunk = u >> 3, unit = u & 7;
-          st_shared_v4(pds_row + chunk * kChunk + ((unit ^ (krow & 7)) << 4), dsk[4 * u], dsk[4 * u + 1],
-                       dsk[4 * u + 2], dsk[4 * u + 3]);
-        }
+        for (int u = 0; u < HC / 8; ++u)
+          st_shared_v4(pds_chunk + ((u ^ (krow & 7)) << 4), dsk[4 * u], dsk[4 * u + 1], dsk[4 * u + 2],
+                       dsk[4 * u + 3]);
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.dst_full);
@@ -687,9 +688,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         __nv_bfloat16* dst = part == 0 ? dv_row : dk_row;
         const float f = part == 0 ? 1.0f : prm.scale;
 #pragma unroll
-        for (int g = 0; g < D / 32; ++g) {
+        for (int g = 0; g < HD / 32; ++g) {
           uint32_t r[32];
-          tmem_ld32(tmem + lane_base + 256 + part * 128 + g * 32, r);
+          tmem_ld32(tmem + lane_base + 256 + part * 128 + half * HD + g * 32, r);
           tmem_wait_ld();
           if (row_ok) {
 #pragma unroll
@@ -725,6 +726,7 @@ size_t attn_bwd_tc_ws(const AttnProblem& p) {
 
 constexpr size_t kMaxDynSmem = 232448;  // 227 KB opt-in per block on sm_100/sm_103
 static_assert(sizeof(DqSmem<128>) <= kMaxDynSmem, "dQ shared layout exceeds the per-block limit");
+static_assert(kDqColDs + kTile / 2 <= 512, "dQ TMEM columns");
 static_assert(sizeof(DkdvSmem<128>) <= kMaxDynSmem, "dK/dV shared layout exceeds the per-block limit");
 
 template <int D>
@@ -738,10 +740,10 @@ static cudaError_t launch_bwd_d(const AttnProblem& p, const CUtensorMap* tm, Bwd
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(bwd_dkdv_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_kv);
   if (e != cudaSuccess) return e;
-  bwd_dkdv_kernel<D><<<grid, kBwdThreads, smem_kv, s>>>(tm[0], tm[1], tm[2], tm[3], prm_kv);
+  bwd_dkdv_kernel<D><<<grid, kDkdvThreads, smem_kv, s>>>(tm[0], tm[1], tm[2], tm[3], prm_kv);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  bwd_dq_kernel<D><<<grid, kBwdThreads, smem_dq, s>>>(tm[0], tm[1], tm[2], tm[3], prm_dq);
+  bwd_dq_kernel<D><<<grid, kDqThreads, smem_dq, s>>>(tm[0], tm[1], tm[2], tm[3], prm_dq);
   return cudaGetLastError();
 }
 

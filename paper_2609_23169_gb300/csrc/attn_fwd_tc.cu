@@ -169,41 +169,47 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         const int L = prm.row_ptr[w + 1] - prm.row_ptr[w];
         if (L <= 0) continue;
         if (!(ok = warp_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        for (int t = 0; t <= L && ok; ++t) {
-          if (t < L) {
-            const uint32_t kv = kv0 + t, st = kv % kStages, n = kv / kStages;
-            const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
-            if (!(ok = warp_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = warp_wait(&sm.s_empty[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            tc_fence_after();
-            const uint32_t k_addr = smem_u32(sm.k[st]);
+        // S runs two key blocks ahead of P V: S_{u+2} goes into the S buffer
+        // that softmax u has just read, so the tensor core computes it while
+        // the softmax works, and PV_u follows as soon as P_u is in TMEM.
+        auto issue_s = [&](int t) -> bool {
+          const uint32_t kv = kv0 + t, st = kv % kStages, n = kv / kStages;
+          const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
+          if (!warp_wait(&sm.k_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+          if (!warp_wait(&sm.s_empty[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+          tc_fence_after();
+          const uint32_t k_addr = smem_u32(sm.k[st]);
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kTileChunkBytes + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem + sb * 128, sdesc_sw128(q_addr + off, 16, 1024),
-                            sdesc_sw128(k_addr + off, 16, 1024), idesc_s, kk > 0);
-            }
-            mma_commit_w(&sm.s_full[sb]);
-            mma_commit_w(&sm.k_empty[st]);
-            if (t == L - 1) mma_commit_w(&sm.q_empty);
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * kTileChunkBytes + (kk & 3) * 32;
+            mma_bf16_ss_w(tmem + sb * 128, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024),
+                          idesc_s, kk > 0);
           }
-          if (t >= 1) {
-            const uint32_t u = t - 1;
-            const uint32_t kv = kv0 + u, st = kv % kStages, n = kv / kStages;
-            const uint32_t sc = sc0 + u, pb = sc & 1, np = sc >> 1;
-            if (!(ok = warp_wait(&sm.p_full[pb], np & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = warp_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (u == 0 && !(ok = warp_wait(&sm.o_empty, (oi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
-              break;
-            tc_fence_after();
-            const uint32_t v_addr = smem_u32(sm.v[st]);
+          mma_commit_w(&sm.s_full[sb]);
+          mma_commit_w(&sm.k_empty[st]);
+          if (t == L - 1) mma_commit_w(&sm.q_empty);
+          return true;
+        };
+        auto issue_pv = [&](int u) -> bool {
+          const uint32_t kv = kv0 + u, st = kv % kStages, n = kv / kStages;
+          const uint32_t sc = sc0 + u, pb = sc & 1, np = sc >> 1;
+          if (!warp_wait(&sm.p_full[pb], np & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+          if (!warp_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+          if (u == 0 && !warp_wait(&sm.o_empty, (oi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+          tc_fence_after();
+          const uint32_t v_addr = smem_u32(sm.v[st]);
 #pragma unroll
-            for (int kk = 0; kk < kBN / 16; ++kk)
-              mma_bf16_ts_w(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
-                            sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024), idesc_o, (u > 0 || kk > 0));
-            mma_commit_w(&sm.pv_done[pb]);
-            mma_commit_w(&sm.v_empty[st]);
-          }
+          for (int kk = 0; kk < kBN / 16; ++kk)
+            mma_bf16_ts_w(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
+                          sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024), idesc_o, (u > 0 || kk > 0));
+          mma_commit_w(&sm.pv_done[pb]);
+          mma_commit_w(&sm.v_empty[st]);
+          return true;
+        };
+        ok = issue_s(0) && (L < 2 || issue_s(1));
+        for (int u = 0; u < L && ok; ++u) {
+          if (u + 2 < L && !(ok = issue_s(u + 2))) break;
+          ok = issue_pv(u);
         }
         kv0 += L;
         sc0 += L;
