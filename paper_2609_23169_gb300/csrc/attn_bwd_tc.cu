@@ -381,21 +381,27 @@ __global__ void __launch_bounds__(kDqThreads, 1)
 // =========================================================================
 //                                dK, dV
 // =========================================================================
+// TMEM columns (512): S^T and then dP^T of a pair share [0,128) (dP^T is
+// computed once S^T has been read), P^T bf16 pairs [128,192), dS^T bf16 pairs
+// [192,256), dV accumulator [256,384), dK accumulator [384,512).  dV += P^T dO
+// and dK += dS^T Q read their A operand from TMEM (TS form).
+constexpr int kKvQStages = 3, kKvDoStages = 2;
+constexpr uint32_t kColSdp = 0, kColPt = 128, kColDst = 192, kColDv = 256, kColDk = 384;
+
 template <int D>
 struct DkdvSmem {
   static constexpr int kC = D / 64;
   static constexpr uint32_t kTileBytes = kTile * D * 2;
   alignas(1024) uint8_t k[kTileBytes];
   alignas(1024) uint8_t v[kTileBytes];
-  alignas(1024) uint8_t q[2][kTileBytes];
-  alignas(1024) uint8_t dout[2][kTileBytes];
-  alignas(1024) uint8_t pds[kTile * kTile * 2];   // P^T, then dS^T, of the current pair
+  alignas(1024) uint8_t q[kKvQStages][kTileBytes];
+  alignas(1024) uint8_t dout[kKvDoStages][kTileBytes];
   alignas(16) float lse2[2][kTile];
   alignas(16) float dsum[2][kTile];
   uint64_t kv_full, kv_empty;
-  uint64_t q_full[2], q_empty[2], do_full[2], do_empty[2];
+  uint64_t q_full[kKvQStages], q_empty[kKvQStages], do_full[kKvDoStages], do_empty[kKvDoStages];
   uint64_t s_full, s_empty, dp_full, dp_empty, pt_full, pt_done, dst_full, ds_done, acc_full, acc_empty, mma_done;
-  uint64_t rowvec_full[2];   // the 128 elementwise threads staged this pair's LSE / D
+  uint64_t rowvec_full[2];   // the elementwise threads staged this pair's LSE / D
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -418,9 +424,11 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(&sm.kv_full, 1);
     mbar_init(&sm.kv_empty, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kKvQStages; ++s) {
       mbar_init(&sm.q_full[s], 1);
       mbar_init(&sm.q_empty[s], 1);
+    }
+    for (int s = 0; s < kKvDoStages; ++s) {
       mbar_init(&sm.do_full[s], 1);
       mbar_init(&sm.do_empty[s], 1);
     }
@@ -467,6 +475,7 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
       uint64_t* empty = is_q ? sm.q_empty : sm.do_empty;
       uint8_t* ring = is_q ? &sm.q[0][0] : &sm.dout[0][0];
       const void* tmap = is_q ? static_cast<const void*>(&tm_q) : static_cast<const void*>(&tm_do);
+      const uint32_t nst = is_q ? kKvQStages : kKvDoStages;
       uint32_t ki = 0, qd = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
@@ -484,8 +493,7 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
         }
         for (int t = 0; t < L; ++t, ++qd) {
           const int i = prm.idx[beg + t];
-          const int st = qd & 1;
-          const uint32_t n = qd >> 1;
+          const uint32_t st = qd % nst, n = qd / nst;
           if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
           mbar_expect_tx(&full[st], TB);
           for (int c = 0; c < C; ++c)
@@ -496,83 +504,77 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
         if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
       };
       if (ki > 0) drain(&sm.kv_full, (ki - 1) & 1);
-      for (uint32_t u = (qd >= 2 ? qd - 2 : 0); u < qd; ++u) drain(&full[u & 1], (u >> 1) & 1);
+      for (uint32_t u = (qd >= nst ? qd - nst : 0); u < qd; ++u) drain(&full[u % nst], (u / nst) & 1);
     }
   } else if (warp == 1) {
-    // whole warp, converged: waits are warp-uniform, MMAs/commits elect one lane
+    // whole warp, converged: waits are warp-uniform, MMAs/commits elect one lane.
+    // Per pair t: dP^T_t (after S^T_t was read), dV_t (after P^T_t is in TMEM),
+    // S^T_{t+1} (after dP^T_t was read), dK_t (after dS^T_t is in TMEM).
     {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
       constexpr uint32_t idesc_acc = idesc_bf16_f32(kTile, D, false, true);
-      const uint32_t k_addr = smem_u32(sm.k), v_addr = smem_u32(sm.v), pds_addr = smem_u32(sm.pds);
+      const uint32_t k_addr = smem_u32(sm.k), v_addr = smem_u32(sm.v);
       uint32_t ki = 0, qd0 = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int L = prm.ptr[w + 1] - prm.ptr[w];
         if (L <= 0) continue;
         if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        for (int t = 0; t <= L && ok; ++t) {
-          // issue order per step: dV_{t-1}, S^T_t, dP^T_t, dK_{t-1} (dV first: it only
-          // needs P^T_{t-1}, so it never waits behind the Q ring)
-          const uint32_t qd_t = qd0 + t, st_t = qd_t & 1, n_t = qd_t >> 1;
-          if (t >= 1) {
-            const uint32_t u = t - 1;
-            const uint32_t qd = qd0 + u, st = qd & 1;
-            const uint32_t do_addr = smem_u32(sm.dout[st]);
-            if (!(ok = warp_wait(&sm.pt_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (u == 0 && !(ok = warp_wait(&sm.acc_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
-              break;
-            tc_fence_after();
+        auto issue_st = [&](int t) -> bool {  // S^T_t = K Q_t^T into [0,128)
+          const uint32_t qd = qd0 + t, st = qd % kKvQStages, n = qd / kKvQStages;
+          if (!warp_wait(&sm.q_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+          if (!warp_wait(&sm.dp_empty, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+          tc_fence_after();
+          const uint32_t q_addr = smem_u32(sm.q[st]);
 #pragma unroll
-            for (int kk = 0; kk < kTile / 16; ++kk) {
-              const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem + 256, sdesc_sw128(pds_addr + aoff, 16, 1024),
-                          sdesc_sw128(do_addr + kk * 2048, kChunk, 1024), idesc_acc, (u > 0 || kk > 0));
-            }
-            mma_commit_w(&sm.pt_done);
-            mma_commit_w(&sm.do_empty[st]);
-          }
-          if (t < L) {
-            if (!(ok = warp_wait(&sm.q_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = warp_wait(&sm.s_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            tc_fence_after();
-            const uint32_t q_addr = smem_u32(sm.q[st_t]);
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024), idesc_s,
-                          kk > 0);
-            }
-            mma_commit_w(&sm.s_full);
-          }
-          if (t < L) {
-            if (!(ok = warp_wait(&sm.do_full[st_t], n_t & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = warp_wait(&sm.dp_empty, (qd_t & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            tc_fence_after();
-            const uint32_t do_addr = smem_u32(sm.dout[st_t]);
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem + 128, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+            mma_bf16_ss_w(tmem + kColSdp, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024),
                           idesc_s, kk > 0);
-            }
-            mma_commit_w(&sm.dp_full);
-            if (t == L - 1) mma_commit_w(&sm.kv_empty);
           }
-          if (t >= 1) {
-            const uint32_t u = t - 1;
-            const uint32_t qd = qd0 + u, st = qd & 1;
-            const uint32_t q_addr = smem_u32(sm.q[st]);
-            if (!(ok = warp_wait(&sm.dst_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            tc_fence_after();
+          mma_commit_w(&sm.s_full);
+          return true;
+        };
+        if (!(ok = issue_st(0))) break;
+        for (int t = 0; t < L && ok; ++t) {
+          const uint32_t qd = qd0 + t;
+          const uint32_t sq = qd % kKvQStages, sd = qd % kKvDoStages, nd = qd / kKvDoStages;
+          // dP^T_t = V dO_t^T into [0,128) once S^T_t has been read
+          if (!(ok = warp_wait(&sm.do_full[sd], nd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          if (!(ok = warp_wait(&sm.s_empty, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          tc_fence_after();
+          const uint32_t do_addr = smem_u32(sm.dout[sd]);
 #pragma unroll
-            for (int kk = 0; kk < kTile / 16; ++kk) {
-              const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem + 384, sdesc_sw128(pds_addr + aoff, 16, 1024),
-                          sdesc_sw128(q_addr + kk * 2048, kChunk, 1024), idesc_acc, (u > 0 || kk > 0));
-            }
-            mma_commit_w(&sm.ds_done);
-            mma_commit_w(&sm.q_empty[st]);
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+            mma_bf16_ss_w(tmem + kColSdp, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
+                          idesc_s, kk > 0);
           }
+          mma_commit_w(&sm.dp_full);
+          if (t == L - 1) mma_commit_w(&sm.kv_empty);
+          // dV += P^T_t dO_t
+          if (!(ok = warp_wait(&sm.pt_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          if (t == 0 && !(ok = warp_wait(&sm.acc_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+            break;
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk)
+            mma_bf16_ts_w(tmem + kColDv, tmem + kColPt + kk * 8, sdesc_sw128(do_addr + kk * 2048, kChunk, 1024),
+                          idesc_acc, (t > 0 || kk > 0));
+          mma_commit_w(&sm.pt_done);
+          mma_commit_w(&sm.do_empty[sd]);
+          // S^T_{t+1} once dP^T_t has been read
+          if (t + 1 < L && !(ok = issue_st(t + 1))) break;
+          // dK += dS^T_t Q_t
+          if (!(ok = warp_wait(&sm.dst_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          tc_fence_after();
+          const uint32_t q_addr = smem_u32(sm.q[sq]);
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk)
+            mma_bf16_ts_w(tmem + kColDk, tmem + kColDst + kk * 8, sdesc_sw128(q_addr + kk * 2048, kChunk, 1024),
+                          idesc_acc, (t > 0 || kk > 0));
+          mma_commit_w(&sm.ds_done);
+          mma_commit_w(&sm.q_empty[sq]);
         }
         mma_commit_w(&sm.acc_full);
         qd0 += L;
@@ -584,8 +586,7 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
   } else {
     // 8 elementwise warps: warps w and w+4 share TMEM lane quarter (w & 3),
     // i.e. the same 32 key rows, and split the 128 query columns (and the D
-    // output columns) into halves.  A half is exactly one 128-byte swizzle
-    // chunk of the shared P^T / dS^T tile.
+    // output columns) into halves.
     const uint32_t quarter = warp & 3;
     const uint32_t half = (warp - 2) >> 2;
     const uint32_t krow = quarter * 32 + lane;          // key row of the tile = TMEM lane
@@ -611,7 +612,6 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
           }
         continue;
       }
-      const uint32_t pds_chunk = smem_u32(sm.pds) + half * kChunk + krow * 128;
       for (int t = 0; t < L; ++t) {
         const uint32_t qd = qd0 + t;
         const int i = prm.idx[beg + t];
@@ -630,7 +630,7 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
         float p[HC];
         {
           uint32_t r[HC];
-          tmem_ld64(tmem + lane_base + half * HC, r);
+          tmem_ld64(tmem + lane_base + kColSdp + half * HC, r);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.s_empty);
@@ -643,25 +643,28 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
             p[x + 3] = ex2_approx(fmaf(__uint_as_float(r[x + 3]), c, -l4.w));
           }
         }
-        // the shared P/dS tile is free once the previous pair's dK MMA finished
-        if (!(ok = warp_wait(&sm.ds_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        {
+          uint32_t pk[HC / 2];
 #pragma unroll
-        for (int u = 0; u < HC / 8; ++u)
-          st_shared_v4(pds_chunk + ((u ^ (krow & 7)) << 4), pack_bf16x2(p[8 * u], p[8 * u + 1]),
-                       pack_bf16x2(p[8 * u + 2], p[8 * u + 3]), pack_bf16x2(p[8 * u + 4], p[8 * u + 5]),
-                       pack_bf16x2(p[8 * u + 6], p[8 * u + 7]));
-        fence_proxy_async_smem();
+          for (int x = 0; x < HC; x += 2) pk[x / 2] = pack_bf16x2(p[x], p[x + 1]);
+          // the TMEM P^T region is free once the previous pair's dV MMA finished
+          if (!(ok = warp_wait(&sm.pt_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          tc_fence_after();
+          tmem_st32(tmem + lane_base + kColPt + half * (HC / 2), pk);
+          tmem_wait_st();
+        }
+        tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.pt_full);
-        uint32_t dsk[HC / 2];
         if (!(ok = warp_wait(&sm.dp_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
         {
           uint32_t r[HC];
-          tmem_ld64(tmem + lane_base + 128 + half * HC, r);
+          tmem_ld64(tmem + lane_base + kColSdp + half * HC, r);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.dp_empty);
+          uint32_t dsk[HC / 2];
 #pragma unroll
           for (int x = 0; x < HC; x += 4) {
             const float4 d4 = *reinterpret_cast<const float4*>(ds_v + x);
@@ -669,14 +672,13 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
             dsk[x / 2 + 1] =
                 pack_bf16x2(p[x + 2] * (__uint_as_float(r[x + 2]) - d4.z), p[x + 3] * (__uint_as_float(r[x + 3]) - d4.w));
           }
+          // the TMEM dS^T region is free once the previous pair's dK MMA finished
+          if (!(ok = warp_wait(&sm.ds_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          tc_fence_after();
+          tmem_st32(tmem + lane_base + kColDst + half * (HC / 2), dsk);
+          tmem_wait_st();
         }
-        // overwrite P^T with dS^T once the dV MMA has read P^T
-        if (!(ok = warp_wait(&sm.pt_done, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-#pragma unroll
-        for (int u = 0; u < HC / 8; ++u)
-          st_shared_v4(pds_chunk + ((u ^ (krow & 7)) << 4), dsk[4 * u], dsk[4 * u + 1], dsk[4 * u + 2],
-                       dsk[4 * u + 3]);
-        fence_proxy_async_smem();
+        tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.dst_full);
       }
@@ -690,7 +692,7 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
 #pragma unroll
         for (int g = 0; g < HD / 32; ++g) {
           uint32_t r[32];
-          tmem_ld32(tmem + lane_base + 256 + part * 128 + half * HD + g * 32, r);
+          tmem_ld32(tmem + lane_base + (part == 0 ? kColDv : kColDk) + half * HD + g * 32, r);
           tmem_wait_ld();
           if (row_ok) {
 #pragma unroll
