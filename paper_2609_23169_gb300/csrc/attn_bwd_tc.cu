@@ -612,15 +612,19 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
           }
         continue;
       }
+      // this thread's element of the query-row vectors (LSE*log2e for threads
+      // 0-127, D for 128-255) is loaded one pair ahead
+      const float* rv_src = (tid < kTile ? prm.lse2 + tid : prm.dsum + (tid - kTile)) + (int64_t)h * prm.Np;
+      float rv = rv_src[(int64_t)prm.idx[beg] * kTile];
       for (int t = 0; t < L; ++t) {
         const uint32_t qd = qd0 + t;
-        const int i = prm.idx[beg + t];
         // this pair's query-row LSE*log2e and D into the shared double buffer
         // (buffer qd&1 was last read in pair qd-2, which every thread finished
         //  before arriving for pair qd-1)
-        if (tid < kTile) sm.lse2[qd & 1][tid] = prm.lse2[(int64_t)h * prm.Np + (int64_t)i * kTile + tid];
-        else sm.dsum[qd & 1][tid - kTile] = prm.dsum[(int64_t)h * prm.Np + (int64_t)i * kTile + tid - kTile];
+        if (tid < kTile) sm.lse2[qd & 1][tid] = rv;
+        else sm.dsum[qd & 1][tid - kTile] = rv;
         mbar_arrive(&sm.rowvec_full[qd & 1]);
+        if (t + 1 < L) rv = rv_src[(int64_t)prm.idx[beg + t + 1] * kTile];
         if (!(ok = warp_wait(&sm.rowvec_full[qd & 1], (qd >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
           break;
         const float* ls = sm.lse2[qd & 1] + half * HC;
@@ -720,16 +724,511 @@ __global__ void __launch_bounds__(kDkdvThreads, 1)
   if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
+// =========================================================================
+//                       fused dK, dV and dQ (one kernel)
+// =========================================================================
+// Item = (head h, key block j); the pairs are the query blocks i of the
+// transposed list.  Per pair, with the 128 key rows as TMEM lanes:
+//   S^T  = K Q_i^T         -> TMEM R0            (A = K, B = Q_i; smem)
+//   P^T  = exp2(S^T c - LSE_i log2 e)   -> bf16, shared tile PT
+//   dP^T = V dO_i^T        -> TMEM R0 (after S^T was read)
+//   dV  += P^T dO_i        (A = PT, B = dO_i)
+//   dS^T = P^T o (dP^T - D_i)           -> bf16, shared tile DST
+//   dK  += dS^T Q_i        (A = DST, B = Q_i)
+//   dQ_i^T = K^T dS^T      -> TMEM RQ            (A = K read d-major, B = DST)
+// and four drain warps add dQ_i^T into an fp32 [H, N_q*128, d] accumulator
+// with coalesced reductions (lane = d, one 128-byte row segment per query
+// row), off the elementwise warps' path; S and dP are computed once per pair.
+// A final kernel scales the accumulator by the softmax scale and writes dQ in
+// bf16.  Roles (512 threads, four warpgroups; the register file is rebalanced
+// with setmaxnreg): warpgroup 0 = warp 0 TMA, warp 1 TMEM owner + MMA issuer
+// (warps 2-3 idle); warpgroups 1-2 = 8 elementwise warps; warpgroup 3 = 4 dQ
+// drain warps.
+// TMEM columns: R0 [0,128), RQ [128,256), dV [256,256+d), dK [384,384+d).
+// For d = 64 the A operand K^T of the dQ product is padded to 128 rows with a
+// zero sub-tile placed right after K, and the padding rows of RQ are ignored.
+constexpr int kFuThreads = 512;
+// registers per thread after setmaxnreg, per warpgroup; the sum equals the
+// launch allocation (4 x 128) so that every increase is covered by decreases
+constexpr int kFuRegLaunch = 128, kFuRegCtl = 96, kFuRegEw = 168, kFuRegDrain = 80;
+static_assert(kFuRegCtl + 2 * kFuRegEw + kFuRegDrain == 4 * kFuRegLaunch, "setmaxnreg split must match the launch");
+// Ring depths: Q is held from S^T to dK (late in the pair), dO only from dP^T
+// to dV (early), so dO gets one stage and its 32 KB buy separate P^T and
+// dS^T tiles: P^T of the next pair never waits for this pair's dK and dQ.
+constexpr int kFuQStages = 2, kFuDoStages = 1;
+constexpr uint32_t kColR0 = 0, kColRQ = 128, kColFuDv = 256, kColFuDk = 384;
+
+template <int D>
+struct FusedSmem {
+  static constexpr int kC = D / 64;
+  static constexpr uint32_t kTileBytes = kTile * D * 2;
+  alignas(1024) uint8_t k[2 * kChunk];        // K (d/64 sub-tiles), then zeros up to 128 d-rows
+  alignas(1024) uint8_t v[kTileBytes];
+  alignas(1024) uint8_t pt[kTile * kTile * 2];   // P^T of the current pair
+  alignas(1024) uint8_t dst[kTile * kTile * 2];  // dS^T of the current pair
+  alignas(1024) uint8_t q[kFuQStages][kTileBytes];
+  alignas(1024) uint8_t dout[kFuDoStages][kTileBytes];
+  alignas(16) float lse2[2][kTile];
+  alignas(16) float dsum[2][kTile];
+  uint64_t kv_full, kv_empty;
+  uint64_t q_full[kFuQStages], q_empty[kFuQStages], do_full[kFuDoStages], do_empty[kFuDoStages];
+  uint64_t s_full, s_empty, dp_full, dp_empty, pt_full, pt_done, dst_full, ds_done, dq_empty;
+  uint64_t acc_full, acc_empty, mma_done;
+  uint64_t rowvec_full[2];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+UT_DEV void red_add_f32(float* p, float v) {
+  asm volatile("red.relaxed.gpu.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
+}
+
+template <int D>
+__global__ void __launch_bounds__(kFuThreads, 1)
+    bwd_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                     const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+                     const BwdParams prm, float* __restrict__ dq_acc) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  FusedSmem<D>& sm = *reinterpret_cast<FusedSmem<D>*>(smem_raw);
+  constexpr int C = FusedSmem<D>::kC;
+  constexpr uint32_t TB = FusedSmem<D>::kTileBytes;
+  const uint32_t warp = warp_id(), lane = lane_id();
+  volatile int* abort_flag = &sm.abort_flag;
+  if ((smem_u32(smem_raw) & 1023u) != 0) {
+    if (threadIdx.x == 0) set_status(prm.status, UT_ERR_INVALID_ARG);
+    return;
+  }
+  if (D == 64) {  // zero padding sub-tile of K^T (rows d = 64..127 of the dQ product)
+    uint4* z = reinterpret_cast<uint4*>(sm.k + kChunk);
+    for (uint32_t x = threadIdx.x; x < kChunk / 16; x += blockDim.x) z[x] = make_uint4(0, 0, 0, 0);
+    fence_proxy_async_smem();
+  }
+  if (threadIdx.x == 0) {
+    mbar_init(&sm.kv_full, 1);
+    mbar_init(&sm.kv_empty, 1);
+    for (int s = 0; s < kFuQStages; ++s) {
+      mbar_init(&sm.q_full[s], 1);
+      mbar_init(&sm.q_empty[s], 1);
+    }
+    for (int s = 0; s < kFuDoStages; ++s) {
+      mbar_init(&sm.do_full[s], 1);
+      mbar_init(&sm.do_empty[s], 1);
+    }
+    mbar_init(&sm.s_full, 1);
+    mbar_init(&sm.s_empty, 8);
+    mbar_init(&sm.dp_full, 1);
+    mbar_init(&sm.dp_empty, 8);
+    mbar_init(&sm.pt_full, 8);
+    mbar_init(&sm.pt_done, 1);
+    mbar_init(&sm.dst_full, 8);
+    mbar_init(&sm.ds_done, 1);
+    mbar_init(&sm.dq_empty, 4);
+    mbar_init(&sm.acc_full, 1);
+    mbar_init(&sm.acc_empty, 8);
+    mbar_init(&sm.mma_done, 1);
+    mbar_init(&sm.rowvec_full[0], 256);
+    mbar_init(&sm.rowvec_full[1], 256);
+    sm.abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  const int G = gridDim.x;
+  const uint32_t wg = warp >> 2;
+  if (wg == 0) {
+    setmaxnreg_dec<kFuRegCtl>();
+    if (warp == 0) {
+      // lane 0: K, V of the item and the Q ring (Q is freed after dK += dS^T Q);
+      // lane 1: the dO ring (dO is freed after dV += P^T dO).
+      if (lane < 2) {
+        const bool is_q = lane == 0;
+        if (is_q) {
+          tma_prefetch_desc(&tm_q);
+          tma_prefetch_desc(&tm_k);
+          tma_prefetch_desc(&tm_v);
+        } else {
+          tma_prefetch_desc(&tm_do);
+        }
+        const uint64_t pol_qd = policy_evict_last(), pol_kv = policy_evict_first();
+        uint64_t* full = is_q ? sm.q_full : sm.do_full;
+        uint64_t* empty = is_q ? sm.q_empty : sm.do_empty;
+        uint8_t* ring = is_q ? &sm.q[0][0] : &sm.dout[0][0];
+        const void* tmap = is_q ? static_cast<const void*>(&tm_q) : static_cast<const void*>(&tm_do);
+        const uint32_t nst = is_q ? kFuQStages : kFuDoStages;
+        uint32_t ki = 0, qd = 0;
+        bool ok = true;
+        for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+          const int h = w / prm.nq, j = w % prm.nq;
+          const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+          if (L <= 0) continue;
+          if (is_q) {
+            if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            mbar_expect_tx(&sm.kv_full, 2 * TB);
+            for (int c = 0; c < C; ++c) {
+              tma_load_2d(sm.k + c * kChunk, &tm_k, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
+              tma_load_2d(sm.v + c * kChunk, &tm_v, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
+            }
+            ++ki;
+          }
+          for (int t = 0; t < L; ++t, ++qd) {
+            const int i = prm.idx[beg + t];
+            const uint32_t st = qd % nst, n = qd / nst;
+            if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            mbar_expect_tx(&full[st], TB);
+            for (int c = 0; c < C; ++c)
+              tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, i * kTile, pol_qd);
+          }
+        }
+        auto drain = [&](uint64_t* bar, uint32_t parity) {
+          if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
+        };
+        if (ki > 0) drain(&sm.kv_full, (ki - 1) & 1);
+        for (uint32_t u = (qd >= nst ? qd - nst : 0); u < qd; ++u) drain(&full[u % nst], (u / nst) & 1);
+      }
+    } else if (warp == 1) {
+      // whole warp, converged: waits are warp-uniform, MMAs/commits elect one lane.
+      // Per pair t: dP^T_t, dV_t, S^T_{t+1}, dK_t, dQ_t^T.
+      {
+        constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
+        constexpr uint32_t idesc_acc = idesc_bf16_f32(kTile, D, false, true);
+        constexpr uint32_t idesc_dq = idesc_bf16_f32(kTile, kTile, true, true);
+        const uint32_t k_addr = smem_u32(sm.k), v_addr = smem_u32(sm.v);
+      const uint32_t pt_addr = smem_u32(sm.pt), dst_addr = smem_u32(sm.dst);
+        uint32_t ki = 0, qd0 = 0;
+        bool ok = true;
+        for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+          const int L = prm.ptr[w + 1] - prm.ptr[w];
+          if (L <= 0) continue;
+          if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+          auto issue_st = [&](int t) -> bool {  // S^T_t = K Q_t^T into R0
+            const uint32_t qd = qd0 + t, st = qd % kFuQStages, n = qd / kFuQStages;
+            if (!warp_wait(&sm.q_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+            if (!warp_wait(&sm.dp_empty, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+            tc_fence_after();
+            const uint32_t q_addr = smem_u32(sm.q[st]);
+  #pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss_w(tmem + kColR0, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024),
+                            idesc_s, kk > 0);
+            }
+            mma_commit_w(&sm.s_full);
+            return true;
+          };
+          if (!(ok = issue_st(0))) break;
+          for (int t = 0; t < L && ok; ++t) {
+            const uint32_t qd = qd0 + t, sq = qd % kFuQStages, sd = qd % kFuDoStages, nd = qd / kFuDoStages;
+            const uint32_t do_addr = smem_u32(sm.dout[sd]), q_addr = smem_u32(sm.q[sq]);
+            // dP^T_t = V dO_t^T into R0 once S^T_t has been read
+            if (!(ok = warp_wait(&sm.do_full[sd], nd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (!(ok = warp_wait(&sm.s_empty, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+  #pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss_w(tmem + kColR0, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
+                            idesc_s, kk > 0);
+            }
+            mma_commit_w(&sm.dp_full);
+            // dV += P^T_t dO_t
+            if (!(ok = warp_wait(&sm.pt_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            if (t == 0 && !(ok = warp_wait(&sm.acc_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+              break;
+            tc_fence_after();
+  #pragma unroll
+            for (int kk = 0; kk < kTile / 16; ++kk) {
+              const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss_w(tmem + kColFuDv, sdesc_sw128(pt_addr + aoff, 16, 1024),
+                            sdesc_sw128(do_addr + kk * 2048, kChunk, 1024), idesc_acc, (t > 0 || kk > 0));
+            }
+            mma_commit_w(&sm.pt_done);
+            mma_commit_w(&sm.do_empty[sd]);
+            // S^T_{t+1} once dP^T_t has been read
+            if (t + 1 < L && !(ok = issue_st(t + 1))) break;
+            // dK += dS^T_t Q_t
+            if (!(ok = warp_wait(&sm.dst_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+  #pragma unroll
+            for (int kk = 0; kk < kTile / 16; ++kk) {
+              const uint32_t aoff = (kk >> 2) * kChunk + (kk & 3) * 32;
+              mma_bf16_ss_w(tmem + kColFuDk, sdesc_sw128(dst_addr + aoff, 16, 1024),
+                            sdesc_sw128(q_addr + kk * 2048, kChunk, 1024), idesc_acc, (t > 0 || kk > 0));
+            }
+            mma_commit_w(&sm.q_empty[sq]);
+            // dQ_t^T = K^T dS^T_t into RQ once the previous pair's dQ^T was drained
+            if (!(ok = warp_wait(&sm.dq_empty, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            tc_fence_after();
+  #pragma unroll
+            for (int kk = 0; kk < kTile / 16; ++kk)
+              mma_bf16_ss_w(tmem + kColRQ, sdesc_sw128(k_addr + kk * 2048, kChunk, 1024),
+                            sdesc_sw128(dst_addr + kk * 2048, kChunk, 1024), idesc_dq, kk > 0);
+            mma_commit_w(&sm.ds_done);
+            if (t == L - 1) mma_commit_w(&sm.kv_empty);
+          }
+          mma_commit_w(&sm.acc_full);
+          qd0 += L;
+          ++ki;
+        }
+        mma_commit_w(&sm.mma_done);
+        if (!mbar_drain(&sm.mma_done, 0, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
+      }
+  }
+  } else if (wg == 1 || wg == 2) {
+    setmaxnreg_inc<kFuRegEw>();
+    // 8 elementwise warps: warps w and w+4 share TMEM lane quarter (w & 3),
+    // i.e. the same 32 key rows, and split the 128 query columns (and the D
+    // output columns) into halves.  A half is exactly one 128-byte swizzle
+    // sub-tile of the shared P^T / dS^T tile.
+    const uint32_t quarter = warp & 3;
+    const uint32_t half = (warp - 4) >> 2;
+    const uint32_t krow = quarter * 32 + lane;  // key row of the tile = TMEM lane (d index for dQ^T)
+    const uint32_t tid = threadIdx.x - 128;     // 0..255 within the elementwise group
+    const uint32_t lane_base = (quarter * 32) << 16;
+    constexpr int HC = kTile / 2;               // query columns per half
+    constexpr int HD = D / 2;                   // output columns per half
+    const float c = prm.scale_log2;
+    const uint32_t pt_row = smem_u32(sm.pt) + half * kChunk + krow * 128;
+    const uint32_t dst_row = smem_u32(sm.dst) + half * kChunk + krow * 128;
+    uint32_t qd0 = 0, ki = 0;
+    bool ok = true;
+    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+      const int h = w / prm.nq, j = w % prm.nq;
+      const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+      const int64_t gk = (int64_t)j * kTile + krow;
+      const bool row_ok = gk < prm.N;
+      __nv_bfloat16* dv_row = prm.out0 + gk * prm.rs + (int64_t)h * D + half * HD;
+      __nv_bfloat16* dk_row = prm.out1 + gk * prm.rs + (int64_t)h * D + half * HD;
+      if (L <= 0) {
+        if (row_ok)
+          for (int e = 0; e < HD; e += 8) {
+            *reinterpret_cast<uint4*>(dv_row + e) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(dk_row + e) = make_uint4(0, 0, 0, 0);
+          }
+        continue;
+      }
+      // this thread's element of the query-row vectors (LSE*log2e for threads
+      // 0-127, D for 128-255) is loaded one pair ahead
+      const float* rv_src = (tid < kTile ? prm.lse2 + tid : prm.dsum + (tid - kTile)) + (int64_t)h * prm.Np;
+      float rv = rv_src[(int64_t)prm.idx[beg] * kTile];
+      for (int t = 0; t < L; ++t) {
+        const uint32_t qd = qd0 + t;
+        // this pair's query-row LSE*log2e and D into the shared double buffer
+        // (buffer qd&1 was last read in pair qd-2, which every thread finished
+        //  before arriving for pair qd-1)
+        if (tid < kTile) sm.lse2[qd & 1][tid] = rv;
+        else sm.dsum[qd & 1][tid - kTile] = rv;
+        mbar_arrive(&sm.rowvec_full[qd & 1]);
+        if (t + 1 < L) rv = rv_src[(int64_t)prm.idx[beg + t + 1] * kTile];
+        if (!(ok = warp_wait(&sm.rowvec_full[qd & 1], (qd >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
+          break;
+        const float* ls = sm.lse2[qd & 1] + half * HC;
+        const float* ds_v = sm.dsum[qd & 1] + half * HC;
+        if (!(ok = warp_wait(&sm.s_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
+        float p[HC];
+        {
+          uint32_t r[HC];
+          tmem_ld64(tmem + lane_base + kColR0 + half * HC, r);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.s_empty);
+#pragma unroll
+          for (int x = 0; x < HC; x += 4) {
+            const float4 l4 = *reinterpret_cast<const float4*>(ls + x);
+            p[x + 0] = ex2_approx(fmaf(__uint_as_float(r[x + 0]), c, -l4.x));
+            p[x + 1] = ex2_approx(fmaf(__uint_as_float(r[x + 1]), c, -l4.y));
+            p[x + 2] = ex2_approx(fmaf(__uint_as_float(r[x + 2]), c, -l4.z));
+            p[x + 3] = ex2_approx(fmaf(__uint_as_float(r[x + 3]), c, -l4.w));
+          }
+        }
+        // the P^T tile is free once the previous pair's dV MMA finished
+        if (!(ok = warp_wait(&sm.pt_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+#pragma unroll
+        for (int u = 0; u < HC / 8; ++u)
+          st_shared_v4(pt_row + ((u ^ (krow & 7)) << 4), pack_bf16x2(p[8 * u], p[8 * u + 1]),
+                       pack_bf16x2(p[8 * u + 2], p[8 * u + 3]), pack_bf16x2(p[8 * u + 4], p[8 * u + 5]),
+                       pack_bf16x2(p[8 * u + 6], p[8 * u + 7]));
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.pt_full);
+        if (!(ok = warp_wait(&sm.dp_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
+        // dS^T in two 32-column steps (fewer live registers); the dS^T tile is
+        // free once the previous pair's dK and dQ^T MMAs finished
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + kColR0 + half * HC + hh * 32, r);
+          tmem_wait_ld();
+          if (hh == 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.dp_empty);
+          }
+          uint32_t dsk[16];
+#pragma unroll
+          for (int x = 0; x < 32; x += 4) {
+            const float4 d4 = *reinterpret_cast<const float4*>(ds_v + hh * 32 + x);
+            const float* pp = p + hh * 32 + x;
+            dsk[x / 2] = pack_bf16x2(pp[0] * (__uint_as_float(r[x]) - d4.x), pp[1] * (__uint_as_float(r[x + 1]) - d4.y));
+            dsk[x / 2 + 1] =
+                pack_bf16x2(pp[2] * (__uint_as_float(r[x + 2]) - d4.z), pp[3] * (__uint_as_float(r[x + 3]) - d4.w));
+          }
+          if (hh == 0 && !(ok = warp_wait(&sm.ds_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
+            break;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int uu = hh * 4 + u;
+            st_shared_v4(dst_row + ((uu ^ (krow & 7)) << 4), dsk[4 * u], dsk[4 * u + 1], dsk[4 * u + 2],
+                         dsk[4 * u + 3]);
+          }
+        }
+        if (!ok) break;
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.dst_full);
+      }
+      if (!ok) break;
+      if (!(ok = warp_wait(&sm.acc_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+      tc_fence_after();
+#pragma unroll
+      for (int part = 0; part < 2; ++part) {
+        __nv_bfloat16* dst = part == 0 ? dv_row : dk_row;
+        const float f = part == 0 ? 1.0f : prm.scale;
+#pragma unroll
+        for (int g = 0; g < HD / 32; ++g) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + (part == 0 ? kColFuDv : kColFuDk) + half * HD + g * 32, r);
+          tmem_wait_ld();
+          if (row_ok) {
+#pragma unroll
+            for (int x = 0; x < 32; x += 8) {
+              uint4 v;
+              v.x = pack_bf16x2(__uint_as_float(r[x + 0]) * f, __uint_as_float(r[x + 1]) * f);
+              v.y = pack_bf16x2(__uint_as_float(r[x + 2]) * f, __uint_as_float(r[x + 3]) * f);
+              v.z = pack_bf16x2(__uint_as_float(r[x + 4]) * f, __uint_as_float(r[x + 5]) * f);
+              v.w = pack_bf16x2(__uint_as_float(r[x + 6]) * f, __uint_as_float(r[x + 7]) * f);
+              *reinterpret_cast<uint4*>(dst + g * 32 + x) = v;
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.acc_empty);
+      qd0 += L;
+      ++ki;
+    }
+  } else {
+    setmaxnreg_dec<kFuRegDrain>();
+    // 4 dQ drain warps, one per TMEM lane quarter: for dQ_i^T the TMEM lane is
+    // the d index.  Each thread adds its d of all 128 query rows of block i,
+    // one fp32 reduction per row; the warp covers 32 consecutive d of a row
+    // (one 128-byte segment).  RQ is released once both halves are read.
+    const uint32_t quarter = warp & 3;
+    const uint32_t dcol = quarter * 32 + lane;
+    const uint32_t lane_base = (quarter * 32) << 16;
+    uint32_t qd0 = 0;
+    bool ok = true;
+    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+      const int h = w / prm.nq;
+      const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+      if (L <= 0) continue;
+      for (int t = 0; t < L; ++t) {
+        const uint32_t qd = qd0 + t;
+        const int i = prm.idx[beg + t];
+        if (!(ok = warp_wait(&sm.ds_done, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        tc_fence_after();
+        float* dst = dq_acc + (((int64_t)h * prm.Np + (int64_t)i * kTile) * D + dcol);
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+          uint32_t r[64];
+          tmem_ld64(tmem + lane_base + kColRQ + g * 64, r);
+          if (g == 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sm.dq_empty);
+          }
+          if (dcol < (uint32_t)D) {
+#pragma unroll
+            for (int x = 0; x < 64; ++x) red_add_f32(dst + (int64_t)(g * 64 + x) * D, __uint_as_float(r[x]));
+          }
+        }
+      }
+      qd0 += L;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// dQ = scale * accumulator, bf16, rows < N: thread = 8 consecutive d of one (row, head)
+__global__ void __launch_bounds__(256) bwd_dq_finalize_kernel(const float* __restrict__ acc, int64_t N, int64_t Np,
+                                                              int H, int d, int64_t rs, float scale,
+                                                              __nv_bfloat16* __restrict__ dq) {
+  const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int per_row = H * d / 8;
+  if (g >= N * per_row) return;
+  const int64_t r = g / per_row;
+  const int e = (int)(g % per_row) * 8;
+  const int h = e / d, c = e % d;
+  const float4* src = reinterpret_cast<const float4*>(acc + ((int64_t)h * Np + r) * d + c);
+  const float4 a = src[0], b = src[1];
+  uint4 v;
+  v.x = pack_bf16x2(a.x * scale, a.y * scale);
+  v.y = pack_bf16x2(a.z * scale, a.w * scale);
+  v.z = pack_bf16x2(b.x * scale, b.y * scale);
+  v.w = pack_bf16x2(b.z * scale, b.w * scale);
+  *reinterpret_cast<uint4*>(dq + r * rs + e) = v;
+}
+
 // ----------------------------------------------------------------- launcher
+// The fused kernel replaces the dQ and dK/dV kernel pair (it computes S and dP
+// once per block pair instead of twice) at the cost of an fp32 dQ accumulator
+// in the workspace.
+constexpr bool kFusedBwd = true;
+
 size_t attn_bwd_tc_ws(const AttnProblem& p) {
   const size_t Np = (size_t)p.nq * kTile;
-  return 2 * (size_t)p.H * Np * sizeof(float);
+  return 2 * (size_t)p.H * Np * sizeof(float) + (kFusedBwd ? (size_t)p.H * Np * p.d * sizeof(float) : 0);
 }
 
 constexpr size_t kMaxDynSmem = 232448;  // 227 KB opt-in per block on sm_100/sm_103
 static_assert(sizeof(DqSmem<128>) <= kMaxDynSmem, "dQ shared layout exceeds the per-block limit");
 static_assert(kDqColDs + kTile / 2 <= 512, "dQ TMEM columns");
 static_assert(sizeof(DkdvSmem<128>) <= kMaxDynSmem, "dK/dV shared layout exceeds the per-block limit");
+static_assert(sizeof(FusedSmem<128>) <= kMaxDynSmem, "fused backward shared layout exceeds the per-block limit");
+
+template <int D>
+static cudaError_t launch_bwd_fused(const AttnProblem& p, const CUtensorMap* tm, BwdParams prm, float* dq_acc,
+                                   __nv_bfloat16* dq, int sms, cudaStream_t s) {
+  const int n_items = p.H * p.nq;
+  const int grid = n_items < sms ? n_items : sms;
+  const size_t smem = sizeof(FusedSmem<D>);
+  cudaError_t e = cudaFuncSetAttribute(bwd_fused_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  // the setmaxnreg split assumes exactly kFuRegLaunch registers per thread at
+  // launch: with fewer, the increases would wait for registers that never come
+  cudaFuncAttributes fa;
+  e = cudaFuncGetAttributes(&fa, bwd_fused_kernel<D>);
+  if (e != cudaSuccess) return e;
+  if (fa.numRegs != kFuRegLaunch) return cudaErrorInvalidConfiguration;
+  bwd_fused_kernel<D><<<grid, kFuThreads, smem, s>>>(tm[0], tm[1], tm[2], tm[3], prm, dq_acc);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int64_t n8 = p.N * p.H * D / 8;
+  bwd_dq_finalize_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, s>>>(dq_acc, p.N, (int64_t)p.nq * kTile, p.H, D,
+                                                                      p.row_stride, p.scale, dq);
+  return cudaGetLastError();
+}
 
 template <int D>
 static cudaError_t launch_bwd_d(const AttnProblem& p, const CUtensorMap* tm, BwdParams prm_dq, BwdParams prm_kv,
@@ -757,6 +1256,11 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
   const int64_t Np = (int64_t)p.nq * kTile;
   float* lse2 = static_cast<float*>(ws);
   float* dsum = lse2 + (size_t)p.H * Np;
+  float* dq_acc = dsum + (size_t)p.H * Np;
+  if (kFusedBwd) {
+    cudaError_t e0 = cudaMemsetAsync(dq_acc, 0, (size_t)p.H * Np * p.d * sizeof(float), stream);
+    if (e0 != cudaSuccess) return e0;
+  }
   bwd_pre_kernel<<<(unsigned)((Np + 7) / 8), 256, 0, stream>>>(
       static_cast<const __nv_bfloat16*>(o), static_cast<const __nv_bfloat16*>(dout), lse, p.N, Np, p.H, p.d,
       p.row_stride, lse2, dsum);
@@ -788,6 +1292,9 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
   pk.idx = row_idx_t;
   pk.out0 = static_cast<__nv_bfloat16*>(dv);
   pk.out1 = static_cast<__nv_bfloat16*>(dk);
+  if (kFusedBwd)
+    return p.d == 64 ? launch_bwd_fused<64>(p, tm, pk, dq_acc, static_cast<__nv_bfloat16*>(dq), sms, stream)
+                     : launch_bwd_fused<128>(p, tm, pk, dq_acc, static_cast<__nv_bfloat16*>(dq), sms, stream);
   return p.d == 64 ? launch_bwd_d<64>(p, tm, pq, pk, sms, stream) : launch_bwd_d<128>(p, tm, pq, pk, sms, stream);
 }
 
