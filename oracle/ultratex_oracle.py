@@ -21,6 +21,11 @@ no blocking, fusion or reordering beyond what the definition states:
 * Scatter back to canvas positions: background rows are "not updated"
   (Sec. 3.2, "Efficient Inference"); ``z_mix`` places foreground latents at
   their positions and a fill elsewhere (Sec. 3.4, the z_mix equation).
+* Sampler steps on the canvas latent: the sparse Euler update (Sec. 3.2,
+  Eq. euler) moves only the retained positions by (t_prev - t_curr) times
+  their predicted velocity; the composite latent (Sec. 3.4, Eq. mixed_latent)
+  keeps the denoised foreground and takes the canonical background latent,
+  tile-repeated over the canvas, everywhere else.
 
 Readings where the paper is silent (listed with the design notes):
 * tiles are ceil-sized; the last tile may be partial (N is rarely a multiple of b);
@@ -72,6 +77,39 @@ def fg_scatter(idx: np.ndarray, src: np.ndarray, dst_in: np.ndarray,
     elif mode == BG_FILL:
         y[...] = np.asarray(fill_row).reshape(y.shape[1:])
     y[np.asarray(idx, dtype=np.int64)] = src
+    return y
+
+
+# ----------------------------------------------------------- sampler steps
+def fg_euler_update(z: np.ndarray, idx: np.ndarray, v: np.ndarray, dt: float) -> np.ndarray:
+    """Sparse Euler step (Sec. 3.2, Eq. euler), in float64.
+
+    ``z``: canvas latent [T, ...]; ``idx``: the retained positions M_fg
+    (distinct); ``v``: predicted velocities of the retained tokens, row n for
+    position idx[n]; ``dt`` = t_prev - t_curr.  z_i <- z_i + dt * v_i for
+    i in M_fg; every other row keeps its value (the background stays at its
+    initial noise).
+    """
+    y = np.array(z, dtype=np.float64, copy=True)
+    ii = np.asarray(idx, dtype=np.int64)
+    y[ii] = y[ii] + float(dt) * np.asarray(v, dtype=np.float64)[: len(ii)]
+    return y
+
+
+def fg_composite(z: np.ndarray, mask: np.ndarray, z_bg_tile: np.ndarray) -> np.ndarray:
+    """Composite latent z_mix (Sec. 3.4, Eq. mixed_latent).
+
+    Foreground rows (mask = 1) keep the denoised latent; background row t takes
+    the canonical background latent tile-repeated over the canvas,
+    ``z_bg_tile[t mod P]`` with P = len(z_bg_tile) rows per tile (one image's
+    latent when P = side^2 and the images are stored one after another).
+    """
+    y = np.array(z, copy=True)
+    tile = np.asarray(z_bg_tile)
+    P = tile.shape[0]
+    for t in range(y.shape[0]):
+        if not mask[t]:
+            y[t] = tile[t % P]
     return y
 
 

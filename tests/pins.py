@@ -321,3 +321,59 @@ def check_subsample_consistency(o, bitmap_to_csr):
         if not (_close(dk, dK[rows, h]) and _close(dv, dV[rows, h])):
             bad.append("bsattn_bwd_dkdv_rows")
     return bad
+
+
+# ------------------------------------------------------------ sampler steps
+def check_sampler(fg_euler_update, fg_composite, fg_scatter, BG_FILL=2):
+    """Pins of the sparse Euler step (Sec. 3.2, Eq. euler) and the composite
+    latent (Sec. 3.4, Eq. mixed_latent)."""
+    bad = []
+    gd = _load("sampler_hand.json")
+    z = np.array(gd["z"], np.float64)
+    dt = gd["t_prev"] - gd["t_curr"]
+    y = fg_euler_update(z, np.array(gd["idx"], np.int32), np.array(gd["v"], np.float64), dt)
+    if not _close(y, gd["euler"]):
+        bad.append("hand Euler step")
+    y = fg_composite(z, np.array(gd["mask"], np.uint8), np.array(gd["tile"], np.float64))
+    if not _close(y, gd["composite"]):
+        bad.append("hand composite")
+    g = np.random.Generator(np.random.PCG64(11))
+    T, C = 203, 6
+    m = (g.random(T) < 0.45).astype(np.uint8)
+    idx = np.nonzero(m)[0].astype(np.int32)
+    z = g.standard_normal((T, C))
+    v = g.standard_normal((len(idx), C))
+    # dt = 0 and v = 0 leave z unchanged
+    if not np.array_equal(fg_euler_update(z, idx, v, 0.0), z):
+        bad.append("Euler with dt = 0 changed z")
+    if not np.array_equal(fg_euler_update(z, idx, np.zeros_like(v), -0.3), z):
+        bad.append("Euler with v = 0 changed z")
+    # background rows are never updated (bit for bit)
+    y = fg_euler_update(z, idx, v, -0.125)
+    if not np.array_equal(y[m == 0], z[m == 0]):
+        bad.append("Euler touched a background row")
+    # a constant velocity field is integrated exactly by Euler: after steps
+    # whose sizes sum to t_end - t_start the foreground moved by that times v
+    steps = [0.25, 0.125, 0.375, 0.25]                       # t: 1 -> 0 (dyadic sizes)
+    y = z.copy()
+    for h in steps:
+        y = fg_euler_update(y, idx, v, -h)
+    if not (np.allclose(y[idx], z[idx] - v, rtol=0, atol=1e-12) and np.array_equal(y[m == 0], z[m == 0])):
+        bad.append("Euler does not integrate a constant velocity exactly")
+    # composite: all-foreground keeps z, all-background is the tile repeated,
+    # foreground rows are bit-exact copies, period 1 equals the FILL scatter
+    P = 17
+    tile = g.standard_normal((P, C))
+    if not np.array_equal(fg_composite(z, np.ones(T, np.uint8), tile), z):
+        bad.append("composite with all foreground is not the identity")
+    allbg = fg_composite(z, np.zeros(T, np.uint8), tile)
+    if not np.array_equal(allbg, np.tile(tile, (-(-T // P), 1))[:T]):
+        bad.append("composite with all background is not the repeated tile")
+    y = fg_composite(z, m, tile)
+    if not np.array_equal(y[m == 1], z[m == 1]):
+        bad.append("composite changed a foreground row")
+    y1 = fg_composite(z, m, tile[:1])
+    yf = fg_scatter(idx, z[idx], z, BG_FILL, tile[0])
+    if not np.array_equal(y1, yf):
+        bad.append("composite with a one-row tile differs from the FILL scatter")
+    return bad

@@ -31,6 +31,10 @@ def test_backward_pinned():
     assert pins.check_backward(o.bsattn_fwd, o.bsattn_bwd, o.bitmap_to_csr) == []
 
 
+def test_sampler_steps_pinned():
+    assert pins.check_sampler(o.fg_euler_update, o.fg_composite, o.fg_scatter) == []
+
+
 def test_row_subset_helpers_agree():
     assert pins.check_subsample_consistency(o, o.bitmap_to_csr) == []
 
@@ -169,6 +173,27 @@ def _scatter_zero_everything(idx, src, dst_in, mode=0, fill_row=None):
     return o.fg_scatter(idx, src, dst_in, o.BG_ZERO, fill_row)
 
 
+def _euler_sign_flipped(z, idx, v, dt):
+    return o.fg_euler_update(z, idx, v, -dt)
+
+
+def _euler_rows_in_order(z, idx, v, dt):
+    return o.fg_euler_update(z, np.arange(len(idx)), v, dt)
+
+
+def _composite_tile_by_block(z, mask, tile):
+    y = np.array(z, copy=True)
+    P = len(tile)
+    for t in range(len(y)):
+        if not mask[t]:
+            y[t] = tile[(t // P) % P]
+    return y
+
+
+def _composite_overwrites_all(z, mask, tile):
+    return o.fg_composite(z, np.zeros_like(mask), tile)
+
+
 def _csr_descending(bm):
     rp, ci = o.bitmap_to_csr(bm)
     ci = ci.copy()
@@ -192,6 +217,12 @@ def _csr_descending(bm):
     ("compaction off by one", lambda: pins.check_compaction(_compact_off_by_one, o.fg_scatter)),
     ("scatter ignores the mode", lambda: pins.check_compaction(o.fg_compact, _scatter_zero_everything)),
     ("CSR lists descending", lambda: pins.check_block_lists(_csr_descending, o.csr_to_csc)),
+    ("Euler step with t_curr - t_prev", lambda: pins.check_sampler(_euler_sign_flipped, o.fg_composite, o.fg_scatter)),
+    ("Euler step on rows 0..n-1", lambda: pins.check_sampler(_euler_rows_in_order, o.fg_composite, o.fg_scatter)),
+    ("composite tile indexed by t // P", lambda: pins.check_sampler(o.fg_euler_update, _composite_tile_by_block,
+                                                                    o.fg_scatter)),
+    ("composite overwrites the foreground", lambda: pins.check_sampler(o.fg_euler_update, _composite_overwrites_all,
+                                                                       o.fg_scatter)),
 ])
 def test_planted_mistake_is_caught(name, check):
     assert check() != [], f"the pins did not catch: {name}"
