@@ -321,6 +321,8 @@ def run_ours(args, rank, world, local_rank):
                                                       (w.T - N) * w.heads * w.head_dim * 2)
     kernels["scatter"]["gbs"] = round(sc_bytes / (kern_ms["scatter"] * 1e-3) / 1e9, 1)
 
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    sampler = time_sampler_steps(w, dev, hbm_peak) if rank == 0 else None
     line = {
         "metric": "retained-block attention TFLOP/s and % of GB300 bf16 peak at 2048 canvas (~213K tokens)",
         "value": round(value, 3),
@@ -350,12 +352,58 @@ def run_ours(args, rank, world, local_rank):
         "gpu_launches": args.steps * hp_launches(hp),
         "clocks": clk,
     }
+    if sampler is not None:
+        line["sampler_steps"] = sampler
     return line, w
+
+
+def time_sampler_steps(w, dev, hbm_peak: float, reps: int = 20) -> dict:
+    """The sampler steps around the model call (sparse Euler update, Eq. euler;
+    composite latent, Eq. mixed_latent), timed alone on the workload's target
+    canvas (bf16, 64 latent channels per token), L2 flushed before each call.
+    Not part of the attention step's time."""
+    import torch
+    from paper_2609_23169_gb300 import ultratex as u
+    x = w.sampler_inputs()
+    mask_np = x["mask"]
+    idx = torch.from_numpy(np.flatnonzero(mask_np).astype(np.int32)).to(dev)
+    n, T = int(idx.numel()), int(mask_np.size)
+    mask = torch.from_numpy(mask_np).to(dev)
+    z, v, tile = x["z"].to(dev), x["v"].to(dev), x["tile"].to(dev)
+    row = z[0].numel() * z.element_size()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    st = u.status_word(dev)
+
+    def timed(fn):
+        fn()
+        tot = 0.0
+        for _ in range(reps):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            tot += e0.elapsed_time(e1)
+        return tot / reps
+
+    ms_e = timed(lambda: u.ut_fg_euler_update(idx, n, z, v, x["dt"], status=st))
+    ms_c = timed(lambda: u.ut_fg_composite(mask, z, tile))
+    u.check_status(st)
+    b_e = n * (4 + 3 * row)            # idx, v read, z read + write (foreground rows)
+    b_c = T + (T - n) * row            # mask read, background rows written
+    out = {"workload": f"{w.name} target canvas: {T} tokens, {n} foreground, 64 channels bf16, "
+                       f"tile of {x['period']} rows", "l2": "flushed before each call"}
+    for name, ms, b in (("euler_update", ms_e, b_e), ("composite", ms_c, b_c)):
+        gbs = b / (ms * 1e-3) / 1e9
+        out[name] = {"ms": round(ms, 5), "bytes": int(b), "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4)}
+    return out
 
 
 def hp_launches(hp) -> int:
     """Kernel launches of one HotPath.step (compaction 3, Top-K lists 3 + transpose 3,
-    forward 1, backward 3 (preprocess, dK/dV, dQ), scatter 2)."""
+    forward 1, backward 3 (preprocess, fused dK/dV/dQ, dQ finalize), scatter 2)."""
     return 3 + 6 + 1 + 3 + 2
 
 

@@ -133,6 +133,42 @@ ut_status ut_fg_scatter(const int32_t* idx, int64_t n, int32_t n_tensors,
                         int32_t bg_mode, const void* fill_row, int64_t T, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Sparse Euler step of the flow-matching sampler (Sec. 3.2, Eq. euler):
+ *   z[idx[n]] += dt * v[n]  for n < n,   dt = t_prev - t_curr,
+ * only at the retained positions; background rows of z are not touched (they
+ * stay at their initial noise, as the paper's inference does).
+ *   idx       [n] int32 canvas positions (as ut_fg_compact writes them);
+ *             distinct, each in [0, T).
+ *   z         [T, channels] canvas latent (dtype), updated in place.
+ *   v         [n, channels] predicted velocities of the retained tokens, row n
+ *             for position idx[n] (dtype).
+ *   channels  latent values per token; channels * element size must be a
+ *             multiple of 16 bytes.
+ *   dtype     UT_BF16 or UT_F32; each element is one fp32 fused multiply-add
+ *             fmaf(dt, v, z) rounded once to dtype (round to nearest even).
+ *   dev_status (may be NULL) receives UT_ERR_INVALID_ARG if an idx value is
+ *             outside [0, T); such rows are skipped.
+ * n = 0 is a no-op.  Host-side argument errors return before any launch. */
+ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T,
+                             int32_t channels, int32_t dtype, float dt, int32_t* dev_status,
+                             void* stream);
+
+/* ------------------------------------------------------------------------
+ * Composite latent for decoding (Sec. 3.4, Eq. mixed_latent):
+ *   z[t] = z_bg[t mod period]  where mask[t] == 0;  foreground rows unchanged.
+ * The canonical background latent (one image's latent, period = its rows;
+ * period = 1 repeats one row everywhere) is tile-repeated over the canvas,
+ * which for images stored one after another in raster order puts tile row
+ * (y, x) at position (y, x) of every image.  A plain bit copy: any dtype.
+ *   mask      [T] uint8, nonzero = foreground (as given to ut_fg_compact).
+ *   z         [T, row_bytes] canvas latent, updated in place.
+ *   z_bg      [period, row_bytes] background tile (device).
+ *   row_bytes a multiple of 16.
+ * T = 0 is a no-op.  Host-side argument errors return before any launch. */
+ut_status ut_fg_composite(const uint8_t* mask, int64_t T, void* z, const void* z_bg, int64_t period,
+                          int64_t row_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
  * Block mask M_c as per-(head, query block) key-block lists (Sec. 3.3).
  * Rows r = h*N_q + i (head-major).  Lists are ascending.
  *

@@ -155,6 +155,28 @@ ut_status ut_fg_scatter(const int32_t* idx, int64_t n, int32_t n_tensors, const 
                                      device_sms(), s));
 }
 
+ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int32_t channels,
+                             int32_t dtype, float dt, int32_t* dev_status, void* stream) {
+  if (n < 0 || T < 0 || n > T || channels <= 0) return UT_ERR_INVALID_ARG;
+  if (dtype != UT_BF16 && dtype != UT_F32) return UT_ERR_INVALID_ARG;
+  const int64_t row_bytes = (int64_t)channels * (dtype == UT_BF16 ? 2 : 4);
+  if (row_bytes % 16 != 0) return UT_ERR_INVALID_ARG;
+  if (!isfinite(dt)) return UT_ERR_INVALID_ARG;
+  if (n == 0) return UT_OK;
+  if (!idx || !z || !v || !aligned16(z) || !aligned16(v)) return UT_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  return from_cuda(launch_fg_euler(idx, n, z, v, T, row_bytes, dtype == UT_BF16, dt, dev_status, device_sms(), s));
+}
+
+ut_status ut_fg_composite(const uint8_t* mask, int64_t T, void* z, const void* z_bg, int64_t period,
+                          int64_t row_bytes, void* stream) {
+  if (T < 0 || period < 1 || row_bytes <= 0 || row_bytes % 16 != 0) return UT_ERR_INVALID_ARG;
+  if (T == 0) return UT_OK;
+  if (!mask || !z || !z_bg || !aligned16(z) || !aligned16(z_bg)) return UT_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  return from_cuda(launch_fg_composite(mask, T, z, z_bg, period, row_bytes, device_sms(), s));
+}
+
 size_t ut_block_mask_workspace_size(const ut_attn_shape* shape, int32_t mode) {
   int nq = 0;
   if (check_shape(shape, &nq) != UT_OK) return 0;

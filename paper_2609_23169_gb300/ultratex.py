@@ -24,7 +24,7 @@ UT_MASK_TOPK, UT_MASK_BITMAP = 0, 1
 EXPORTS = (
     "ut_strerror", "ut_topk_count", "ut_fg_compact_workspace_size", "ut_fg_compact", "ut_fg_scatter",
     "ut_block_mask_workspace_size", "ut_block_mask", "ut_bsattn_fwd", "ut_bsattn_bwd_workspace_size",
-    "ut_bsattn_bwd", "ut_fg_compact_noalloc",
+    "ut_bsattn_bwd", "ut_fg_compact_noalloc", "ut_fg_euler_update", "ut_fg_composite",
 )
 
 
@@ -75,6 +75,10 @@ def lib() -> ctypes.CDLL:
     L.ut_bsattn_bwd.restype = _i32
     L.ut_bsattn_bwd.argtypes = [ctypes.POINTER(AttnShape), _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _flt,
                                 _vp, _vp, _vp, _vp, _sz, _vp, _vp]
+    L.ut_fg_euler_update.restype = _i32
+    L.ut_fg_euler_update.argtypes = [_vp, _i64, _vp, _vp, _i64, _i32, _i32, _flt, _vp, _vp]
+    L.ut_fg_composite.restype = _i32
+    L.ut_fg_composite.argtypes = [_vp, _i64, _vp, _vp, _i64, _i64, _vp]
     _lib = L
     return L
 
@@ -190,6 +194,35 @@ def ut_fg_scatter(idx: torch.Tensor, n: int, srcs: Sequence[torch.Tensor], dsts:
     st = lib().ut_fg_scatter(_p(idx), int(n), len(srcs), _ptr_array(srcs), _ptr_array(dsts), row_bytes, bg_mode,
                              _p(fill_row), T, _stream())
     _check("ut_fg_scatter", st)
+
+
+def ut_fg_euler_update(idx: torch.Tensor, n: int, z: torch.Tensor, v: torch.Tensor, dt: float,
+                       status: Optional[torch.Tensor] = None) -> None:
+    """Sparse Euler step in place: z[idx[i]] += dt * v[i] for i < n (dt = t_prev - t_curr)."""
+    if z.dtype not in (torch.bfloat16, torch.float32) or v.dtype != z.dtype:
+        raise ValueError("z and v must share dtype bf16 or fp32")
+    if not (z.is_contiguous() and v.is_contiguous()):
+        raise ValueError("z and v must be contiguous")
+    T = z.shape[0]
+    C = z[0].numel() if T > 0 else (v[0].numel() if v.shape[0] > 0 else 0)
+    if (v.shape[0] > 0 and v[0].numel() != C) or v.shape[0] < int(n) or idx.numel() < int(n):
+        raise ValueError("v must hold n rows of z's row size; idx n entries")
+    dtype = UT_BF16 if z.dtype == torch.bfloat16 else UT_F32
+    st = lib().ut_fg_euler_update(_p(idx), int(n), _p(z), _p(v), T, C, dtype, float(dt), _p(status), _stream())
+    _check("ut_fg_euler_update", st)
+
+
+def ut_fg_composite(mask: torch.Tensor, z: torch.Tensor, z_bg: torch.Tensor) -> None:
+    """Composite latent in place: background row t of z becomes z_bg[t % len(z_bg)]."""
+    if not (z.is_contiguous() and z_bg.is_contiguous()):
+        raise ValueError("z and z_bg must be contiguous")
+    T = z.shape[0]
+    row_bytes = z[0].numel() * z.element_size() if T > 0 else 0
+    P = z_bg.shape[0]
+    if P < 1 or z_bg[0].numel() * z_bg.element_size() != row_bytes or mask.numel() < T:
+        raise ValueError("z_bg must hold rows of z's row size; mask T entries")
+    st = lib().ut_fg_composite(_p(mask), T, _p(z), _p(z_bg), P, row_bytes, _stream())
+    _check("ut_fg_composite", st)
 
 
 def ut_block_mask(shape: AttnShape, mode: int, q: Optional[torch.Tensor] = None, k: Optional[torch.Tensor] = None,

@@ -16,7 +16,8 @@ Compression").  Images are laid out one after another on the canvas, raster
 order inside each image.
 
 Random streams (numpy PCG64 seeded with ``[seed, stream]``):
-mask=0, Q=1, K=2, V=3, dO=4, block fill=5, oracle row subsample=6.
+mask=0, Q=1, K=2, V=3, dO=4, block fill=5, oracle row subsample=6, sampler
+latent=7, sampler velocity=8, background latent tile=9.
 Q/K/V/dO are drawn N(0,1) in fp32 and, for bf16 workloads, rounded to
 nearest-even bf16 by torch.
 """
@@ -30,6 +31,12 @@ import numpy as np
 import torch
 
 STREAM_MASK, STREAM_Q, STREAM_K, STREAM_V, STREAM_DO, STREAM_FILL, STREAM_ROWS = range(7)
+STREAM_LATENT, STREAM_VEL, STREAM_BG = 7, 8, 9
+
+# Sampler-side latent: 16 VAE channels per 8x8 pixels, 2x2-patchified into one
+# token, i.e. 64 values per token; one step of a 28-step uniform schedule.
+LATENT_CHANNELS = 64
+EULER_DT = -1.0 / 28.0
 
 # The multi-view layout: images 0-5 targets, 6-11 conditions, 12 reference.
 N_VIEWS = 6
@@ -179,6 +186,26 @@ class Workload:
 
     def dout(self) -> torch.Tensor:
         return self._draw(STREAM_DO)
+
+    # ----------------------------------------------------- sampler inputs
+    def sampler_inputs(self, channels: int = LATENT_CHANNELS, dtype: torch.dtype = torch.bfloat16) -> dict:
+        """Inputs of the sampler steps on the target canvas (the noisy target
+        images only: the first six images of the multi-view canvas, or the whole
+        canvas otherwise): its foreground mask, the canvas latent z (Gaussian
+        noise), the predicted velocities of its retained tokens, one image's
+        canonical background latent tile, and the step dt = t_prev - t_curr."""
+        n_img = N_VIEWS if self.multiview else self.n_images
+        T = n_img * self.tokens_per_image
+        mask = self.canvas_mask()[:T].copy()
+        n = int(mask.sum())
+        z = rng(self.seed, STREAM_LATENT).standard_normal((T, channels), dtype=np.float32)
+        v = rng(self.seed, STREAM_VEL).standard_normal((n, channels), dtype=np.float32)
+        gb = rng(self.seed, STREAM_BG)
+        tile = (gb.standard_normal((1, channels), dtype=np.float32) +
+                np.float32(0.1) * gb.standard_normal((self.tokens_per_image, channels), dtype=np.float32))
+        conv = lambda a: torch.from_numpy(a).to(dtype)
+        return {"mask": mask, "z": conv(z), "v": conv(v), "tile": conv(tile), "dt": EULER_DT,
+                "period": self.tokens_per_image}
 
     # ------------------------------------------------- structured block bitmap
     def tile_images(self) -> list[tuple[int, int]]:

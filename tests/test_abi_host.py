@@ -95,6 +95,30 @@ def test_argument_errors_are_caught_on_host(L):
                            bogus, bogus, bogus, bogus, 1 << 20, None, None) == u.UT_ERR_INVALID_ARG
 
 
+def test_sampler_argument_errors_are_caught_on_host(L):
+    from paper_2609_23169_gb300 import ultratex as u
+    bogus = ctypes.c_void_p(16 * 1024)   # never dereferenced: every call must fail validation first
+    odd = ctypes.c_void_p(16 * 1024 + 4)
+    f = L.ut_fg_euler_update
+    # n > T, negative sizes, unknown dtype, rows not a multiple of 16 bytes, non-finite dt, misaligned z
+    assert f(bogus, 11, bogus, bogus, 10, 64, u.UT_BF16, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert f(bogus, -1, bogus, bogus, 10, 64, u.UT_BF16, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert f(bogus, 5, bogus, bogus, 10, 64, 7, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert f(bogus, 5, bogus, bogus, 10, 12, u.UT_BF16, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert f(bogus, 5, bogus, bogus, 10, 6, u.UT_F32, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert f(bogus, 5, bogus, bogus, 10, 64, u.UT_F32, float("nan"), None, None) == u.UT_ERR_INVALID_ARG
+    assert f(bogus, 5, odd, bogus, 10, 64, u.UT_F32, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert f(None, 5, bogus, bogus, 10, 64, u.UT_F32, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    # n = 0 is a no-op (nothing is dereferenced)
+    assert f(None, 0, None, None, 10, 64, u.UT_BF16, 0.5, None, None) == u.UT_OK
+    g = L.ut_fg_composite
+    assert g(bogus, 10, bogus, bogus, 0, 128, None) == u.UT_ERR_INVALID_ARG      # empty tile
+    assert g(bogus, 10, bogus, bogus, 4, 100, None) == u.UT_ERR_INVALID_ARG      # row not 16-byte multiple
+    assert g(bogus, 10, odd, bogus, 4, 128, None) == u.UT_ERR_INVALID_ARG        # misaligned z
+    assert g(None, 10, bogus, bogus, 4, 128, None) == u.UT_ERR_INVALID_ARG       # no mask
+    assert g(None, 0, None, None, 4, 128, None) == u.UT_OK                       # T = 0 is a no-op
+
+
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     from paper_2609_23169_gb300 import ultratex as u
     monkeypatch.setattr(u, "_lib", None)
