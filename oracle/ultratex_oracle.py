@@ -21,6 +21,14 @@ no blocking, fusion or reordering beyond what the definition states:
 * Scatter back to canvas positions: background rows are "not updated"
   (Sec. 3.2, "Efficient Inference"); ``z_mix`` places foreground latents at
   their positions and a fill elsewhere (Sec. 3.4, the z_mix equation).
+* Rotary position embedding at the retained tokens' original canvas positions
+  (Sec. 3.2: each retained token carries its original RoPE index).  The paper
+  does not print the formula; the reading used: canvas position t of images of
+  side S maps to (image, y, x) = (t // S^2, (t mod S^2) // S, t mod S); the
+  head dimension is split into three axes (default 16/56/56 of 128); within
+  axis a of d_a dimensions, pair k = (x[2k], x[2k+1]) is rotated by the angle
+  pos_a * theta^(-2k/d_a) (theta = 10000).  Gathering Q and K applies the
+  rotation; scattering their gradients back applies its inverse.
 * Sampler steps on the canvas latent: the sparse Euler update (Sec. 3.2,
   Eq. euler) moves only the retained positions by (t_prev - t_curr) times
   their predicted velocity; the composite latent (Sec. 3.4, Eq. mixed_latent)
@@ -78,6 +86,62 @@ def fg_scatter(idx: np.ndarray, src: np.ndarray, dst_in: np.ndarray,
         y[...] = np.asarray(fill_row).reshape(y.shape[1:])
     y[np.asarray(idx, dtype=np.int64)] = src
     return y
+
+
+# --------------------------------------------------------------------- RoPE
+def rope_positions(idx: np.ndarray, side: int) -> np.ndarray:
+    """Canvas positions -> (image, y, x) of images of side x side tokens, stored
+    one after another in raster order.  [n] -> [n, 3] int64."""
+    t = np.asarray(idx, dtype=np.int64)
+    s2 = int(side) * int(side)
+    return np.stack([t // s2, (t % s2) // side, t % side], axis=1)
+
+
+def rope_angles(pos: np.ndarray, head_dim: int, axes=(16, 56, 56), theta: float = 10000.0) -> np.ndarray:
+    """Rotation angle of every pair: [n, 3] positions -> [n, head_dim // 2].
+
+    Pairs are taken axis by axis: the first axes[0] / 2 pairs use the image
+    index, the next axes[1] / 2 the row y, the last axes[2] / 2 the column x;
+    pair k of axis a (d_a = axes[a] dimensions) turns by pos_a * theta^(-2k/d_a).
+    """
+    assert sum(axes) == head_dim and all(a % 2 == 0 for a in axes)
+    pos = np.asarray(pos, dtype=np.float64)
+    cols = []
+    for a, d_a in enumerate(axes):
+        k = np.arange(d_a // 2, dtype=np.float64)
+        freq = float(theta) ** (-2.0 * k / d_a)
+        cols.append(pos[:, a:a + 1] * freq[None, :])
+    return np.concatenate(cols, axis=1)
+
+
+def rope_rotate(x: np.ndarray, angles: np.ndarray, inverse: bool = False) -> np.ndarray:
+    """Rotate each consecutive pair (x[..., 2k], x[..., 2k+1]) of every row by
+    angles[row, k] (by -angles[row, k] if ``inverse``).  x: [n, H, d]."""
+    x = np.asarray(x, dtype=np.float64)
+    a = -angles if inverse else angles
+    c = np.cos(a)[:, None, :]
+    s = np.sin(a)[:, None, :]
+    x0, x1 = x[..., 0::2], x[..., 1::2]
+    y = np.empty_like(x)
+    y[..., 0::2] = x0 * c - x1 * s
+    y[..., 1::2] = x0 * s + x1 * c
+    return y
+
+
+def fg_compact_rope(mask: np.ndarray, x: np.ndarray, side: int, axes=(16, 56, 56), theta: float = 10000.0):
+    """Gather of Q or K (Sec. 3.2) with the rotary embedding of each retained
+    token's original canvas position applied.  Returns (idx, rotated rows)."""
+    idx, (xc,) = fg_compact(mask, [x])
+    ang = rope_angles(rope_positions(idx, side), np.asarray(x).shape[-1], axes, theta)
+    return idx, rope_rotate(xc, ang)
+
+
+def fg_scatter_rope(idx: np.ndarray, src: np.ndarray, dst_in: np.ndarray, side: int, mode: int = BG_ZERO,
+                    axes=(16, 56, 56), theta: float = 10000.0) -> np.ndarray:
+    """Scatter of dQ or dK back to the canvas through the inverse rotation (the
+    gradient of the rotated gather); background rows per ``mode``."""
+    ang = rope_angles(rope_positions(idx, side), np.asarray(src).shape[-1], axes, theta)
+    return fg_scatter(idx, rope_rotate(src, ang, inverse=True), dst_in, mode)
 
 
 # ----------------------------------------------------------- sampler steps

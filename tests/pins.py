@@ -377,3 +377,64 @@ def check_sampler(fg_euler_update, fg_composite, fg_scatter, BG_FILL=2):
     if not np.array_equal(y1, yf):
         bad.append("composite with a one-row tile differs from the FILL scatter")
     return bad
+
+
+# --------------------------------------------------------------------- RoPE
+def check_rope(o):
+    """Pins of the rotary embedding at original canvas positions (Sec. 3.2)."""
+    bad = []
+    gd = _load("rope_hand.json")
+    for c in gd["cases"]:
+        pos = o.rope_positions(np.array([c["t"]]), c["side"])
+        if list(pos[0]) != c["pos"]:
+            bad.append(f"hand position of t={c['t']}")
+        ang = o.rope_angles(pos, len(c["x"]), tuple(c["axes"]), c["theta"])
+        if not _close(ang[0], c["angles"]):
+            bad.append(f"hand angles of t={c['t']}")
+        y = o.rope_rotate(np.array(c["x"], np.float64)[None, None, :], ang)[0, 0]
+        if not _close(y, c["y"]):
+            bad.append(f"hand rotation of t={c['t']}")
+    g = np.random.Generator(np.random.PCG64(13))
+    side, H, d = 8, 3, 128
+    T = 5 * side * side
+    idx = np.sort(g.choice(T, size=70, replace=False)).astype(np.int32)
+    x = g.standard_normal((len(idx), H, d))
+    ang = o.rope_angles(o.rope_positions(idx, side), d)
+    y = o.rope_rotate(x, ang)
+    # a rotation keeps every pair's length; the inverse undoes it
+    if not np.allclose(np.hypot(y[..., 0::2], y[..., 1::2]), np.hypot(x[..., 0::2], x[..., 1::2]), atol=1e-12):
+        bad.append("rotation changes a pair's length")
+    if not np.allclose(o.rope_rotate(y, ang, inverse=True), x, atol=1e-12):
+        bad.append("inverse rotation does not undo the rotation")
+    # position (0, 0, 0) is the identity
+    if not np.array_equal(o.rope_rotate(x[:1], o.rope_angles(np.zeros((1, 3)), d)), x[:1]):
+        bad.append("position 0 is not the identity")
+    # the same rotation as complex multiplication (x0 + i x1) e^{i phi}
+    zc = (x[..., 0::2] + 1j * x[..., 1::2]) * np.exp(1j * ang)[:, None, :]
+    if not (np.allclose(y[..., 0::2], zc.real, atol=1e-12) and np.allclose(y[..., 1::2], zc.imag, atol=1e-12)):
+        bad.append("rotation differs from the complex-number form")
+    # the defining RoPE property: q.k after rotation depends only on the
+    # position difference, axis by axis
+    q, k = g.standard_normal(d), g.standard_normal(d)
+    for shift in ([1, 0, 0], [0, 3, 0], [0, 0, 5], [2, 1, 4]):
+        pm, pn = np.array([[1, 2, 3]]), np.array([[4, 6, 1]])
+        s_ = np.array([shift])
+        dots = []
+        for a, b in ((pm, pn), (pm + s_, pn + s_)):
+            rq = o.rope_rotate(q[None, None], o.rope_angles(a, d))[0, 0]
+            rk = o.rope_rotate(k[None, None], o.rope_angles(b, d))[0, 0]
+            dots.append(float(rq @ rk))
+        if abs(dots[0] - dots[1]) > 1e-9 * (1 + abs(dots[0])):
+            bad.append(f"q.k not shift-invariant for shift {shift}")
+    # the gather applies the rotation of each token's own canvas position;
+    # the scatter of the gathered rows through the inverse returns the canvas
+    xt = g.standard_normal((T, H, d))
+    m = np.zeros(T, np.uint8)
+    m[idx] = 1
+    i2, xr = o.fg_compact_rope(m, xt, side)
+    if not (np.array_equal(i2, idx) and np.allclose(xr, o.rope_rotate(xt[idx], ang), atol=1e-12)):
+        bad.append("rope gather is not gather + rotation")
+    back = o.fg_scatter_rope(idx, xr, np.zeros_like(xt), side, o.BG_ZERO)
+    if not (np.allclose(back[idx], xt[idx], atol=1e-12) and not back[m == 0].any()):
+        bad.append("rope scatter is not the inverse of the rope gather")
+    return bad

@@ -35,6 +35,10 @@ def test_sampler_steps_pinned():
     assert pins.check_sampler(o.fg_euler_update, o.fg_composite, o.fg_scatter) == []
 
 
+def test_rope_pinned():
+    assert pins.check_rope(o) == []
+
+
 def test_row_subset_helpers_agree():
     assert pins.check_subsample_consistency(o, o.bitmap_to_csr) == []
 
@@ -194,6 +198,44 @@ def _composite_overwrites_all(z, mask, tile):
     return o.fg_composite(z, np.zeros_like(mask), tile)
 
 
+class _OracleWith:
+    """The oracle module with one function replaced (a planted mistake)."""
+    def __init__(self, **kw):
+        self.__dict__.update(kw)
+
+    def __getattr__(self, name):
+        return getattr(o, name)
+
+
+def _rope_sin_sign(x, angles, inverse=False):
+    return o.rope_rotate(x, -angles, inverse)
+
+
+def _rope_half_split(x, angles, inverse=False):
+    x = np.asarray(x, dtype=np.float64)
+    h = x.shape[-1] // 2
+    a = -angles if inverse else angles
+    c, s_ = np.cos(a)[:, None, :], np.sin(a)[:, None, :]
+    y = np.empty_like(x)
+    y[..., :h] = x[..., :h] * c - x[..., h:] * s_
+    y[..., h:] = x[..., :h] * s_ + x[..., h:] * c
+    return y
+
+
+def _rope_freq_k_over_d(pos, head_dim, axes=(16, 56, 56), theta=10000.0):
+    pos = np.asarray(pos, dtype=np.float64)
+    cols = []
+    for a, d_a in enumerate(axes):
+        k = np.arange(d_a // 2, dtype=np.float64)
+        cols.append(pos[:, a:a + 1] * (float(theta) ** (-k / d_a))[None, :])
+    return np.concatenate(cols, axis=1)
+
+
+def _rope_xy_swapped(idx, side):
+    p = o.rope_positions(idx, side)
+    return p[:, [0, 2, 1]]
+
+
 def _csr_descending(bm):
     rp, ci = o.bitmap_to_csr(bm)
     ci = ci.copy()
@@ -217,6 +259,10 @@ def _csr_descending(bm):
     ("compaction off by one", lambda: pins.check_compaction(_compact_off_by_one, o.fg_scatter)),
     ("scatter ignores the mode", lambda: pins.check_compaction(o.fg_compact, _scatter_zero_everything)),
     ("CSR lists descending", lambda: pins.check_block_lists(_csr_descending, o.csr_to_csc)),
+    ("RoPE with the sine's sign flipped", lambda: pins.check_rope(_OracleWith(rope_rotate=_rope_sin_sign))),
+    ("RoPE pairing halves instead of neighbours", lambda: pins.check_rope(_OracleWith(rope_rotate=_rope_half_split))),
+    ("RoPE frequencies theta^(-k/d)", lambda: pins.check_rope(_OracleWith(rope_angles=_rope_freq_k_over_d))),
+    ("RoPE with x and y swapped", lambda: pins.check_rope(_OracleWith(rope_positions=_rope_xy_swapped))),
     ("Euler step with t_curr - t_prev", lambda: pins.check_sampler(_euler_sign_flipped, o.fg_composite, o.fg_scatter)),
     ("Euler step on rows 0..n-1", lambda: pins.check_sampler(_euler_rows_in_order, o.fg_composite, o.fg_scatter)),
     ("composite tile indexed by t // P", lambda: pins.check_sampler(o.fg_euler_update, _composite_tile_by_block,
