@@ -323,6 +323,7 @@ def run_ours(args, rank, world, local_rank):
 
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
     sampler = time_sampler_steps(w, dev, hbm_peak) if rank == 0 else None
+    rope = time_rope(w, dev, hbm_peak) if rank == 0 else None
     line = {
         "metric": "retained-block attention TFLOP/s and % of GB300 bf16 peak at 2048 canvas (~213K tokens)",
         "value": round(value, 3),
@@ -354,13 +355,16 @@ def run_ours(args, rank, world, local_rank):
     }
     if sampler is not None:
         line["sampler_steps"] = sampler
+    if rope is not None:
+        line["rope_fused"] = rope
     return line, w
 
 
 def time_sampler_steps(w, dev, hbm_peak: float, reps: int = 20) -> dict:
     """The sampler steps around the model call (sparse Euler update, Eq. euler;
     composite latent, Eq. mixed_latent), timed alone on the workload's target
-    canvas (bf16, 64 latent channels per token), L2 flushed before each call.
+    canvas (bf16, 64 latent channels per token), L2 flushed (by a read) before
+    each call.
     Not part of the attention step's time."""
     import torch
     from paper_2609_23169_gb300 import ultratex as u
@@ -371,14 +375,16 @@ def time_sampler_steps(w, dev, hbm_peak: float, reps: int = 20) -> dict:
     mask = torch.from_numpy(mask_np).to(dev)
     z, v, tile = x["z"].to(dev), x["v"].to(dev), x["tile"].to(dev)
     row = z[0].numel() * z.element_size()
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    # L2 is flushed by reading a buffer twice its size: the lines left behind
+    # are clean, so the timed call pays no write-back of someone else's data
+    flush = torch.ones(64 << 20, dtype=torch.float32, device=dev)
     st = u.status_word(dev)
 
     def timed(fn):
         fn()
         tot = 0.0
         for _ in range(reps):
-            flush.zero_()
+            flush.sum()
             e0 = torch.cuda.Event(enable_timing=True)
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record()
@@ -394,10 +400,51 @@ def time_sampler_steps(w, dev, hbm_peak: float, reps: int = 20) -> dict:
     b_e = n * (4 + 3 * row)            # idx, v read, z read + write (foreground rows)
     b_c = T + (T - n) * row            # mask read, background rows written
     out = {"workload": f"{w.name} target canvas: {T} tokens, {n} foreground, 64 channels bf16, "
-                       f"tile of {x['period']} rows", "l2": "flushed before each call"}
+                       f"tile of {x['period']} rows", "l2": "flushed before each call by reading 256 MB"}
     for name, ms, b in (("euler_update", ms_e, b_e), ("composite", ms_c, b_c)):
         gbs = b / (ms * 1e-3) / 1e9
         out[name] = {"ms": round(ms, 5), "bytes": int(b), "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4)}
+    return out
+
+
+def time_rope(w, dev, hbm_peak: float, reps: int = 10) -> dict:
+    """RoPE fused with the gather of Q and K (and, inverted, with the ZERO
+    scatter of dQ and dK) on the workload's canvas; inputs larger than L2.
+    Not part of the attention step's time."""
+    import torch
+    from paper_2609_23169_gb300 import ultratex as u
+    mask = w.canvas_mask()
+    idx = torch.from_numpy(np.flatnonzero(mask).astype(np.int32)).to(dev)
+    N, T = int(idx.numel()), int(mask.size)
+    q, k = w.q().to(dev), w.k().to(dev)
+    cfg = u.rope_config(w.side)
+    qc, kc = (torch.empty((N, w.heads, w.head_dim), dtype=q.dtype, device=dev) for _ in range(2))
+    dq, dk = torch.empty_like(q), torch.empty_like(k)
+    row = w.heads * w.head_dim * q.element_size()
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    ms_g = timed(lambda: u.ut_fg_gather_rope(idx, N, [q, k], cfg, dsts=[qc, kc]))
+    ms_s = timed(lambda: u.ut_fg_scatter_rope(idx, N, [qc, kc], [dq, dk], cfg, u.UT_BG_ZERO))
+    b_g = 2 * 2 * N * row + 4 * N          # read N canvas rows, write N rows, per tensor; idx once
+    b_s = 2 * (N * row + T * row) + 4 * N  # read N rows, write all T canvas rows, per tensor
+    out = {"workload": f"{w.name}: Q and K (H={w.heads}, d={w.head_dim}, bf16), N={N} of T={T} rows, "
+                       f"axes 16/56/56, theta 1e4", "l2": "inputs larger than L2 (1.31 GB per canvas tensor)"}
+    for name, ms, b in (("gather_rope", ms_g, b_g), ("scatter_rope_zero", ms_s, b_s)):
+        gbs = b / (ms * 1e-3) / 1e9
+        out[name] = {"ms": round(ms, 4), "bytes": int(b), "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4)}
+    del q, k, qc, kc, dq, dk
+    torch.cuda.empty_cache()
     return out
 
 

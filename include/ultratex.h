@@ -133,6 +133,47 @@ ut_status ut_fg_scatter(const int32_t* idx, int64_t n, int32_t n_tensors,
                         int32_t bg_mode, const void* fill_row, int64_t T, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Rotary position embedding fused with the gather of Q / K and with the
+ * scatter of dQ / dK (Sec. 3.2: every retained token keeps its original RoPE
+ * index, its canvas position).  The paper does not print the formula; this
+ * library's reading: canvas position t of images of rope->side tokens per side,
+ * stored one after another in raster order, has the coordinates
+ *   (image, y, x) = (t / side^2, (t mod side^2) / side, t mod side);
+ * the head dimension is split into three axes of rope->axes[0..2] dimensions
+ * (even, summing to head_dim; 16/56/56 for 128); pair k of axis a, the
+ * elements (2j, 2j+1) of the head vector, is rotated by the angle
+ * coordinate_a * theta^(-2k/axes[a]).  Angles are formed in fp32 from
+ * frequencies computed in double precision; sin/cos in fp32; the rotated pair
+ * is rounded once to dtype. */
+typedef struct {
+  int32_t side;     /* tokens per image side */
+  int32_t axes[3];  /* head dimensions of the image, y and x axes */
+  float theta;      /* frequency base (10000) */
+} ut_rope;
+
+/* dst[n] = R(idx[n]) src[idx[n]] for n < n, every listed tensor (Q and K):
+ * the gather of ut_fg_compact with the rotation applied, reusing the idx a
+ * ut_fg_compact call wrote (for V, dO).
+ *   src, dst   arrays of n_tensors (1..8) device pointers; src rows [T, H, d],
+ *              dst rows [n, H, d], row = heads * head_dim elements of dtype.
+ *   head_dim   head_dim * element size must divide 512 bytes and be a
+ *              multiple of 16 (bf16: 8..256, fp32: 4..128).
+ * idx values outside [0, T) are skipped.  n = 0 is a no-op. */
+ut_status ut_fg_gather_rope(const int32_t* idx, int64_t n, int32_t n_tensors,
+                            const void* const* h_src, void* const* h_dst, int64_t T,
+                            int32_t heads, int32_t head_dim, int32_t dtype, const ut_rope* rope,
+                            void* stream);
+
+/* The gradient of ut_fg_gather_rope: dst[idx[n]] = R(idx[n])^T src[n] (the
+ * inverse rotation), background rows per bg_mode: UT_BG_KEEP (not written)
+ * or UT_BG_ZERO (set to zero: the adjoint of the gather).  idx strictly
+ * increasing and < T (as ut_fg_compact writes it).  Same layouts as above. */
+ut_status ut_fg_scatter_rope(const int32_t* idx, int64_t n, int32_t n_tensors,
+                             const void* const* h_src, void* const* h_dst, int64_t T,
+                             int32_t heads, int32_t head_dim, int32_t dtype, const ut_rope* rope,
+                             int32_t bg_mode, void* stream);
+
+/* ------------------------------------------------------------------------
  * Sparse Euler step of the flow-matching sampler (Sec. 3.2, Eq. euler):
  *   z[idx[n]] += dt * v[n]  for n < n,   dt = t_prev - t_curr,
  * only at the retained positions; background rows of z are not touched (they

@@ -155,6 +155,51 @@ ut_status ut_fg_scatter(const int32_t* idx, int64_t n, int32_t n_tensors, const 
                                      device_sms(), s));
 }
 
+static ut_status check_rope(int64_t n, int64_t T, int32_t n_tensors, const void* const* h_src,
+                            void* const* h_dst, int32_t heads, int32_t head_dim, int32_t dtype, const ut_rope* rope,
+                            bool gather) {
+  if (n < 0 || T < 0 || n > T || n_tensors < 1 || n_tensors > 8 || heads < 1 || head_dim < 2) return UT_ERR_INVALID_ARG;
+  if (dtype != UT_BF16 && dtype != UT_F32) return UT_ERR_INVALID_ARG;
+  if (!rope || !h_src || !h_dst || rope->side < 1 || !(rope->theta > 0.0f) || !isfinite(rope->theta))
+    return UT_ERR_INVALID_ARG;
+  if (rope->axes[0] < 0 || rope->axes[1] < 0 || rope->axes[2] < 0 || rope->axes[0] % 2 || rope->axes[1] % 2 ||
+      rope->axes[2] % 2 || (int64_t)rope->axes[0] + rope->axes[1] + rope->axes[2] != head_dim)
+    return UT_ERR_INVALID_ARG;
+  const int64_t head_bytes = (int64_t)head_dim * (dtype == UT_BF16 ? 2 : 4);
+  if (head_bytes % 16 != 0 || 512 % head_bytes != 0) return UT_ERR_UNSUPPORTED;
+  for (int i = 0; i < n_tensors; ++i) {
+    const void* rows_n = gather ? h_dst[i] : h_src[i];
+    const void* rows_t = gather ? h_src[i] : h_dst[i];
+    if (n > 0 && (!rows_n || !aligned16(rows_n))) return UT_ERR_INVALID_ARG;
+    if (T > 0 && (!rows_t || !aligned16(rows_t))) return UT_ERR_INVALID_ARG;
+  }
+  return UT_OK;
+}
+
+ut_status ut_fg_gather_rope(const int32_t* idx, int64_t n, int32_t n_tensors, const void* const* h_src,
+                            void* const* h_dst, int64_t T, int32_t heads, int32_t head_dim, int32_t dtype,
+                            const ut_rope* rope, void* stream) {
+  ut_status st = check_rope(n, T, n_tensors, h_src, h_dst, heads, head_dim, dtype, rope, true);
+  if (st != UT_OK) return st;
+  if (n == 0) return UT_OK;
+  if (!idx) return UT_ERR_INVALID_ARG;
+  return from_cuda(launch_fg_rope(idx, n, n_tensors, h_src, h_dst, heads, head_dim, dtype == UT_BF16, rope->side,
+                                  rope->axes, rope->theta, 0, T, device_sms(), static_cast<cudaStream_t>(stream)));
+}
+
+ut_status ut_fg_scatter_rope(const int32_t* idx, int64_t n, int32_t n_tensors, const void* const* h_src,
+                             void* const* h_dst, int64_t T, int32_t heads, int32_t head_dim, int32_t dtype,
+                             const ut_rope* rope, int32_t bg_mode, void* stream) {
+  ut_status st = check_rope(n, T, n_tensors, h_src, h_dst, heads, head_dim, dtype, rope, false);
+  if (st != UT_OK) return st;
+  if (bg_mode != UT_BG_KEEP && bg_mode != UT_BG_ZERO) return UT_ERR_INVALID_ARG;
+  if (n > 0 && !idx) return UT_ERR_INVALID_ARG;
+  const int mode = bg_mode == UT_BG_KEEP ? 1 : 2;
+  if ((mode == 1 && n == 0) || T == 0) return UT_OK;
+  return from_cuda(launch_fg_rope(idx, n, n_tensors, h_src, h_dst, heads, head_dim, dtype == UT_BF16, rope->side,
+                                  rope->axes, rope->theta, mode, T, device_sms(), static_cast<cudaStream_t>(stream)));
+}
+
 ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int32_t channels,
                              int32_t dtype, float dt, int32_t* dev_status, void* stream) {
   if (n < 0 || T < 0 || n > T || channels <= 0) return UT_ERR_INVALID_ARG;

@@ -22,6 +22,11 @@ cudaError_t launch_fg_euler(const int32_t* idx, int64_t n, void* z, const void* 
 cudaError_t launch_fg_composite(const uint8_t* mask, int64_t T, void* z, const void* tile, int64_t period,
                                 int64_t row_bytes, int sms, cudaStream_t stream);
 
+// rope.cu (mode: 0 gather, 1 scatter keeping the background, 2 scatter zeroing it)
+cudaError_t launch_fg_rope(const int32_t* idx, int64_t n, int n_tensors, const void* const* src, void* const* dst,
+                           int heads, int head_dim, bool bf16, int side, const int32_t axes[3], float theta,
+                           int mode, int64_t T, int sms, cudaStream_t stream);
+
 // blockmask.cu
 struct MaskProblem {
   int64_t N;

@@ -25,6 +25,7 @@ EXPORTS = (
     "ut_strerror", "ut_topk_count", "ut_fg_compact_workspace_size", "ut_fg_compact", "ut_fg_scatter",
     "ut_block_mask_workspace_size", "ut_block_mask", "ut_bsattn_fwd", "ut_bsattn_bwd_workspace_size",
     "ut_bsattn_bwd", "ut_fg_compact_noalloc", "ut_fg_euler_update", "ut_fg_composite",
+    "ut_fg_gather_rope", "ut_fg_scatter_rope",
 )
 
 
@@ -37,6 +38,15 @@ class UtError(RuntimeError):
 class AttnShape(ctypes.Structure):
     _fields_ = [("n_tokens", ctypes.c_int64), ("n_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("block", ctypes.c_int32), ("dtype", ctypes.c_int32), ("row_stride", ctypes.c_int64)]
+
+
+class Rope(ctypes.Structure):
+    """ut_rope: tokens per image side, head dimensions of the image / y / x axes, frequency base."""
+    _fields_ = [("side", ctypes.c_int32), ("axes", ctypes.c_int32 * 3), ("theta", ctypes.c_float)]
+
+
+def rope_config(side: int, axes=(16, 56, 56), theta: float = 10000.0) -> Rope:
+    return Rope(int(side), (ctypes.c_int32 * 3)(*axes), float(theta))
 
 
 _lib = None
@@ -79,6 +89,11 @@ def lib() -> ctypes.CDLL:
     L.ut_fg_euler_update.argtypes = [_vp, _i64, _vp, _vp, _i64, _i32, _i32, _flt, _vp, _vp]
     L.ut_fg_composite.restype = _i32
     L.ut_fg_composite.argtypes = [_vp, _i64, _vp, _vp, _i64, _i64, _vp]
+    L.ut_fg_gather_rope.restype = _i32
+    L.ut_fg_gather_rope.argtypes = [_vp, _i64, _i32, _ptrs, _ptrs, _i64, _i32, _i32, _i32, ctypes.POINTER(Rope), _vp]
+    L.ut_fg_scatter_rope.restype = _i32
+    L.ut_fg_scatter_rope.argtypes = [_vp, _i64, _i32, _ptrs, _ptrs, _i64, _i32, _i32, _i32, ctypes.POINTER(Rope),
+                                     _i32, _vp]
     _lib = L
     return L
 
@@ -194,6 +209,44 @@ def ut_fg_scatter(idx: torch.Tensor, n: int, srcs: Sequence[torch.Tensor], dsts:
     st = lib().ut_fg_scatter(_p(idx), int(n), len(srcs), _ptr_array(srcs), _ptr_array(dsts), row_bytes, bg_mode,
                              _p(fill_row), T, _stream())
     _check("ut_fg_scatter", st)
+
+
+def _rope_dims(ts: Sequence[torch.Tensor]):
+    t0 = ts[0]
+    if t0.dim() != 3 or t0.dtype not in (torch.bfloat16, torch.float32):
+        raise ValueError("RoPE tensors are [rows, heads, head_dim] bf16 or fp32")
+    for t in ts:
+        if t.dim() != 3 or t.shape[1:] != t0.shape[1:] or t.dtype != t0.dtype or not t.is_contiguous():
+            raise ValueError("RoPE tensors must share heads, head_dim and dtype, contiguous")
+    return t0.shape[1], t0.shape[2], (UT_BF16 if t0.dtype == torch.bfloat16 else UT_F32)
+
+
+def ut_fg_gather_rope(idx: torch.Tensor, n: int, srcs: Sequence[torch.Tensor], rope: Rope,
+                      dsts: Optional[Sequence[torch.Tensor]] = None):
+    """Rotated gather: dst[i] = R(idx[i]) src[idx[i]] for i < n.  Returns the dst list."""
+    H, d, dtype = _rope_dims(srcs)
+    if dsts is None:
+        dsts = [torch.empty((max(int(n), 1), H, d), dtype=s.dtype, device=s.device) for s in srcs]
+    _rope_dims(list(srcs) + list(dsts))
+    T = srcs[0].shape[0]
+    if any(s.shape[0] != T for s in srcs) or any(t.shape[0] < int(n) for t in dsts) or idx.numel() < int(n):
+        raise ValueError("srcs share T rows; dsts hold n rows; idx n entries")
+    st = lib().ut_fg_gather_rope(_p(idx), int(n), len(srcs), _ptr_array(srcs), _ptr_array(dsts), T, H, d, dtype,
+                                 ctypes.byref(rope), _stream())
+    _check("ut_fg_gather_rope", st)
+    return dsts
+
+
+def ut_fg_scatter_rope(idx: torch.Tensor, n: int, srcs: Sequence[torch.Tensor], dsts: Sequence[torch.Tensor],
+                       rope: Rope, bg_mode: int = UT_BG_ZERO) -> None:
+    """Inverse-rotated scatter: dst[idx[i]] = R(idx[i])^T src[i]; background rows per bg_mode (KEEP / ZERO)."""
+    H, d, dtype = _rope_dims(list(srcs) + list(dsts))
+    T = dsts[0].shape[0]
+    if any(t.shape[0] != T for t in dsts) or any(s.shape[0] < int(n) for s in srcs) or idx.numel() < int(n):
+        raise ValueError("dsts share T rows; srcs hold n rows; idx n entries")
+    st = lib().ut_fg_scatter_rope(_p(idx), int(n), len(srcs), _ptr_array(srcs), _ptr_array(dsts), T, H, d, dtype,
+                                  ctypes.byref(rope), bg_mode, _stream())
+    _check("ut_fg_scatter_rope", st)
 
 
 def ut_fg_euler_update(idx: torch.Tensor, n: int, z: torch.Tensor, v: torch.Tensor, dt: float,

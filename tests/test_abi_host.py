@@ -119,6 +119,31 @@ def test_sampler_argument_errors_are_caught_on_host(L):
     assert g(None, 0, None, None, 4, 128, None) == u.UT_OK                       # T = 0 is a no-op
 
 
+def test_rope_argument_errors_are_caught_on_host(L):
+    from paper_2609_23169_gb300 import ultratex as u
+    bogus = ctypes.c_void_p(16 * 1024)   # never dereferenced: every call must fail validation first
+    arr = (ctypes.c_void_p * 2)(bogus.value, bogus.value)
+    S = ctypes.byref
+    ok = u.rope_config(16)
+    g, sc = L.ut_fg_gather_rope, L.ut_fg_scatter_rope
+    assert g(bogus, 11, 1, arr, arr, 10, 2, 128, u.UT_BF16, S(ok), None) == u.UT_ERR_INVALID_ARG        # n > T
+    assert g(bogus, 5, 9, arr, arr, 10, 2, 128, u.UT_BF16, S(ok), None) == u.UT_ERR_INVALID_ARG         # 9 tensors
+    assert g(bogus, 5, 1, arr, arr, 10, 2, 128, 5, S(ok), None) == u.UT_ERR_INVALID_ARG                 # dtype
+    assert g(bogus, 5, 1, arr, arr, 10, 2, 128, u.UT_BF16, None, None) == u.UT_ERR_INVALID_ARG          # no config
+    assert g(bogus, 5, 1, arr, arr, 10, 2, 120, u.UT_BF16, S(ok), None) == u.UT_ERR_INVALID_ARG         # axes != d
+    assert g(bogus, 5, 1, arr, arr, 10, 2, 128, u.UT_BF16, S(u.rope_config(16, (15, 57, 56))), None) \
+        == u.UT_ERR_INVALID_ARG                                                                         # odd axis
+    assert g(bogus, 5, 1, arr, arr, 10, 2, 128, u.UT_BF16, S(u.rope_config(0)), None) == u.UT_ERR_INVALID_ARG
+    assert g(bogus, 5, 1, arr, arr, 10, 2, 128, u.UT_BF16, S(u.rope_config(16, theta=-1.0)), None) \
+        == u.UT_ERR_INVALID_ARG
+    assert g(bogus, 5, 1, arr, arr, 10, 2, 12, u.UT_BF16, S(u.rope_config(16, (4, 4, 4))), None) \
+        == u.UT_ERR_UNSUPPORTED                                                                         # 24-byte heads
+    assert g(bogus, 5, 1, arr, arr, 10, 2, 96, u.UT_BF16, S(u.rope_config(16, (16, 40, 40))), None) \
+        == u.UT_ERR_UNSUPPORTED                                                                         # 192 B !| 512
+    assert sc(bogus, 5, 1, arr, arr, 10, 2, 128, u.UT_BF16, S(ok), u.UT_BG_FILL, None) == u.UT_ERR_INVALID_ARG
+    assert g(None, 0, 1, arr, arr, 10, 2, 128, u.UT_BF16, S(ok), None) == u.UT_OK                       # n = 0
+
+
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     from paper_2609_23169_gb300 import ultratex as u
     monkeypatch.setattr(u, "_lib", None)
