@@ -21,6 +21,11 @@ no blocking, fusion or reordering beyond what the definition states:
 * Scatter back to canvas positions: background rows are "not updated"
   (Sec. 3.2, "Efficient Inference"); ``z_mix`` places foreground latents at
   their positions and a fill elsewhere (Sec. 3.4, the z_mix equation).
+* Mask construction (Sec. 3.2): a token is foreground when any alpha pixel of
+  its factor x factor block exceeds the threshold (the 1/16 downsampling of
+  the alpha channel), then the token mask is dilated by a square of radius r
+  (the slight dilation); the six view masks serve both the noisy targets and
+  the conditions, the reference image has its own.
 * Rotary position embedding at the retained tokens' original canvas positions
   (Sec. 3.2: each retained token carries its original RoPE index).  The paper
   does not print the formula; the reading used: canvas position t of images of
@@ -86,6 +91,39 @@ def fg_scatter(idx: np.ndarray, src: np.ndarray, dst_in: np.ndarray,
         y[...] = np.asarray(fill_row).reshape(y.shape[1:])
     y[np.asarray(idx, dtype=np.int64)] = src
     return y
+
+
+# ----------------------------------------------------------- mask from alpha
+def token_mask_from_alpha(alpha: np.ndarray, factor: int = 16, radius: int = 1, threshold: int = 0) -> np.ndarray:
+    """One image's token mask (Sec. 3.2): [H_px, W_px] alpha -> [H_px/factor, W_px/factor] uint8.
+
+    Token (y, x) is foreground before dilation when some pixel of its block
+    alpha[y*f:(y+1)*f, x*f:(x+1)*f] exceeds ``threshold``; after dilation when
+    some token within Chebyshev distance ``radius`` (inside the image) is.
+    """
+    a = np.asarray(alpha)
+    h, w = a.shape[0] // factor, a.shape[1] // factor
+    pooled = np.zeros((h, w), dtype=bool)
+    for y in range(h):
+        for x in range(w):
+            pooled[y, x] = bool((a[y * factor:(y + 1) * factor, x * factor:(x + 1) * factor] > threshold).any())
+    out = np.zeros((h, w), dtype=bool)
+    for y in range(h):
+        for x in range(w):
+            out[y, x] = pooled[max(0, y - radius):y + radius + 1, max(0, x - radius):x + radius + 1].any()
+    return out.astype(np.uint8)
+
+
+def canvas_mask_from_alpha(alpha: np.ndarray, factor: int = 16, radius: int = 1, threshold: int = 0) -> np.ndarray:
+    """Canvas mask of the multi-view sequence (Sec. 3.2): alpha [V + 1, H_px, W_px]
+    (V view renders, then the reference) -> [(2V + 1) * h * w] uint8 laid out as
+    the V target images, the V condition images (view v's mask again) and the
+    reference image, raster order inside each."""
+    a = np.asarray(alpha)
+    V = a.shape[0] - 1
+    views = [token_mask_from_alpha(a[v], factor, radius, threshold).ravel() for v in range(V)]
+    ref = token_mask_from_alpha(a[V], factor, radius, threshold).ravel()
+    return np.concatenate(views + views + [ref]).astype(np.uint8)
 
 
 # --------------------------------------------------------------------- RoPE

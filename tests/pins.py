@@ -438,3 +438,58 @@ def check_rope(o):
     if not (np.allclose(back[idx], xt[idx], atol=1e-12) and not back[m == 0].any()):
         bad.append("rope scatter is not the inverse of the rope gather")
     return bad
+
+
+# --------------------------------------------------------- mask from alpha
+def check_alpha_mask(token_mask_from_alpha, canvas_mask_from_alpha):
+    """Pins of the mask construction (Sec. 3.2)."""
+    import scipy.ndimage as ndi
+    bad = []
+    gd = _load("alpha_mask_hand.json")
+    a = np.array(gd["alpha"], np.uint8)
+    if token_mask_from_alpha(a, gd["factor"], 0, gd["threshold"]).tolist() != gd["pooled"]:
+        bad.append("hand pooled mask")
+    if token_mask_from_alpha(a, gd["factor"], gd["radius"], gd["threshold"]).tolist() != gd["dilated"]:
+        bad.append("hand dilated mask")
+    g = np.random.Generator(np.random.PCG64(17))
+    f, H, W = 4, 48, 40
+    alpha = (g.random((H, W)) < 0.02).astype(np.uint8) * g.integers(1, 256, size=(H, W), dtype=np.uint8)
+    # library routines: block any-pool by reshape, square dilation by scipy
+    for thr in (0, 100):
+        pooled = (alpha.reshape(H // f, f, W // f, f) > thr).any(axis=(1, 3))
+        for r in (0, 1, 2):
+            ref = ndi.binary_dilation(pooled, structure=np.ones((2 * r + 1, 2 * r + 1), bool)) if r else pooled
+            if not np.array_equal(token_mask_from_alpha(alpha, f, r, thr), ref.astype(np.uint8)):
+                bad.append(f"differs from pool + scipy dilation (threshold {thr}, radius {r})")
+    # a single lit pixel lights a (2r+1)^2 square of tokens, clipped at the border
+    one = np.zeros((H, W), np.uint8)
+    one[f * 5 + 1, f * 0 + 2] = 255
+    m = token_mask_from_alpha(one, f, 2, 0)
+    sq = np.zeros_like(m)
+    sq[3:8, 0:3] = 1
+    if not np.array_equal(m, sq):
+        bad.append("single pixel is not a clipped square")
+    # empty and full alpha; monotone in the alpha
+    if token_mask_from_alpha(np.zeros((H, W), np.uint8), f, 1, 0).any():
+        bad.append("empty alpha gives foreground")
+    if not token_mask_from_alpha(np.full((H, W), 255, np.uint8), f, 1, 0).all():
+        bad.append("full alpha is not all foreground")
+    more = np.maximum(alpha, (g.random((H, W)) < 0.01).astype(np.uint8) * 255)
+    if np.any(token_mask_from_alpha(alpha, f, 1, 0) > token_mask_from_alpha(more, f, 1, 0)):
+        bad.append("more alpha gives less foreground")
+    # canvas: V targets, the same V masks for the conditions, then the reference
+    V = 3
+    stack = (g.random((V + 1, H, W)) < 0.01).astype(np.uint8) * 255
+    cm = canvas_mask_from_alpha(stack, f, 1, 0)
+    n_tok = (H // f) * (W // f)
+    if cm.size != (2 * V + 1) * n_tok:
+        bad.append("canvas mask size")
+    else:
+        blocks = cm.reshape(2 * V + 1, n_tok)
+        for v in range(V):
+            mv = token_mask_from_alpha(stack[v], f, 1, 0).ravel()
+            if not (np.array_equal(blocks[v], mv) and np.array_equal(blocks[V + v], mv)):
+                bad.append(f"view {v}: target / condition masks")
+        if not np.array_equal(blocks[2 * V], token_mask_from_alpha(stack[V], f, 1, 0).ravel()):
+            bad.append("reference mask")
+    return bad

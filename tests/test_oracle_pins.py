@@ -35,6 +35,10 @@ def test_sampler_steps_pinned():
     assert pins.check_sampler(o.fg_euler_update, o.fg_composite, o.fg_scatter) == []
 
 
+def test_alpha_mask_pinned():
+    assert pins.check_alpha_mask(o.token_mask_from_alpha, o.canvas_mask_from_alpha) == []
+
+
 def test_rope_pinned():
     assert pins.check_rope(o) == []
 
@@ -236,6 +240,29 @@ def _rope_xy_swapped(idx, side):
     return p[:, [0, 2, 1]]
 
 
+def _alpha_all_pixels(alpha, factor=16, radius=1, threshold=0):
+    a = np.asarray(alpha)
+    h, w = a.shape[0] // factor, a.shape[1] // factor
+    pooled = (a.reshape(h, factor, w, factor) > threshold).all(axis=(1, 3))
+    return o.token_mask_from_alpha(pooled.astype(np.uint8) * 255, 1, radius, 0)
+
+
+def _alpha_radius_plus_one(alpha, factor=16, radius=1, threshold=0):
+    return o.token_mask_from_alpha(alpha, factor, radius + 1, threshold)
+
+
+def _alpha_at_least(alpha, factor=16, radius=1, threshold=0):
+    return o.token_mask_from_alpha(alpha, factor, radius, max(threshold - 1, -1))
+
+
+def _canvas_conditions_use_reference(alpha, factor=16, radius=1, threshold=0):
+    a = np.asarray(alpha)
+    V = a.shape[0] - 1
+    views = [o.token_mask_from_alpha(a[v], factor, radius, threshold).ravel() for v in range(V)]
+    ref = o.token_mask_from_alpha(a[V], factor, radius, threshold).ravel()
+    return np.concatenate(views + [ref] * V + [ref]).astype(np.uint8)
+
+
 def _csr_descending(bm):
     rp, ci = o.bitmap_to_csr(bm)
     ci = ci.copy()
@@ -259,6 +286,14 @@ def _csr_descending(bm):
     ("compaction off by one", lambda: pins.check_compaction(_compact_off_by_one, o.fg_scatter)),
     ("scatter ignores the mode", lambda: pins.check_compaction(o.fg_compact, _scatter_zero_everything)),
     ("CSR lists descending", lambda: pins.check_block_lists(_csr_descending, o.csr_to_csc)),
+    ("alpha pooled with all() instead of any()", lambda: pins.check_alpha_mask(_alpha_all_pixels,
+                                                                               o.canvas_mask_from_alpha)),
+    ("alpha dilation one token too wide", lambda: pins.check_alpha_mask(_alpha_radius_plus_one,
+                                                                        o.canvas_mask_from_alpha)),
+    ("alpha compared with >= instead of >", lambda: pins.check_alpha_mask(_alpha_at_least,
+                                                                          o.canvas_mask_from_alpha)),
+    ("conditions take the reference mask", lambda: pins.check_alpha_mask(o.token_mask_from_alpha,
+                                                                         _canvas_conditions_use_reference)),
     ("RoPE with the sine's sign flipped", lambda: pins.check_rope(_OracleWith(rope_rotate=_rope_sin_sign))),
     ("RoPE pairing halves instead of neighbours", lambda: pins.check_rope(_OracleWith(rope_rotate=_rope_half_split))),
     ("RoPE frequencies theta^(-k/d)", lambda: pins.check_rope(_OracleWith(rope_angles=_rope_freq_k_over_d))),
