@@ -133,6 +133,26 @@ ut_status ut_fg_scatter(const int32_t* idx, int64_t n, int32_t n_tensors,
                         int32_t bg_mode, const void* fill_row, int64_t T, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Canvas mask from the renders' alpha channels (Sec. 3.2, mask construction):
+ * the alpha is downsampled to the token grid (a token is foreground when some
+ * pixel of its factor x factor block has alpha > threshold; factor 16 at 8x
+ * VAE downsampling and 2x2 patches) and the token mask is dilated by a square
+ * of radius tokens (radius 1: 3 x 3).  The view masks serve both the noisy
+ * targets and the conditions; the reference image has its own.
+ *   alpha        [n_views + 1, height, width] uint8 (the views, then the
+ *                reference), device.
+ *   canvas_mask  [(2 n_views + 1) * (height/factor) * (width/factor)] uint8
+ *                output, 0/1, laid out as ut_fg_compact expects it: the
+ *                n_views targets, the n_views conditions (view v's mask
+ *                again), the reference; raster order inside each image.
+ *   factor       >= 1, dividing height and width; radius 0..16; threshold
+ *                0..255.
+ * Host-side argument errors return before any launch. */
+ut_status ut_fg_mask_from_alpha(const uint8_t* alpha, int32_t n_views, int32_t height, int32_t width,
+                                int32_t factor, int32_t radius, int32_t threshold, uint8_t* canvas_mask,
+                                void* stream);
+
+/* ------------------------------------------------------------------------
  * Rotary position embedding fused with the gather of Q / K and with the
  * scatter of dQ / dK (Sec. 3.2: every retained token keeps its original RoPE
  * index, its canvas position).  The paper does not print the formula; this

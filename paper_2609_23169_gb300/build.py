@@ -17,7 +17,7 @@ LIBDIR = os.path.join(PKG, "lib")
 OBJDIR = os.path.join(PKG, "_build")
 LIB = os.path.join(LIBDIR, "libultratex.so")
 SOURCES = ["api.cu", "compact.cu", "blockmask.cu", "attn_simt.cu", "attn_fwd_tc.cu", "attn_bwd_tc.cu",
-           "compact_noalloc.cu", "sampler.cu", "rope.cu"]
+           "compact_noalloc.cu", "sampler.cu", "rope.cu", "mask_alpha.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-Xptxas", "-warn-spills"]

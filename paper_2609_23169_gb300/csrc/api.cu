@@ -155,6 +155,20 @@ ut_status ut_fg_scatter(const int32_t* idx, int64_t n, int32_t n_tensors, const 
                                      device_sms(), s));
 }
 
+ut_status ut_fg_mask_from_alpha(const uint8_t* alpha, int32_t n_views, int32_t height, int32_t width,
+                                int32_t factor, int32_t radius, int32_t threshold, uint8_t* canvas_mask,
+                                void* stream) {
+  if (n_views < 0 || height < 0 || width < 0 || factor < 1 || radius < 0 || radius > 16 || threshold < 0 ||
+      threshold > 255)
+    return UT_ERR_INVALID_ARG;
+  if (height % factor != 0 || width % factor != 0) return UT_ERR_INVALID_ARG;
+  if ((int64_t)height * width * (n_views + 1) > ((int64_t)1 << 40)) return UT_ERR_UNSUPPORTED;
+  if (height == 0 || width == 0) return UT_OK;
+  if (!alpha || !canvas_mask) return UT_ERR_INVALID_ARG;
+  return from_cuda(launch_mask_from_alpha(alpha, n_views, height, width, factor, radius, threshold, canvas_mask,
+                                          static_cast<cudaStream_t>(stream)));
+}
+
 static ut_status check_rope(int64_t n, int64_t T, int32_t n_tensors, const void* const* h_src,
                             void* const* h_dst, int32_t heads, int32_t head_dim, int32_t dtype, const ut_rope* rope,
                             bool gather) {

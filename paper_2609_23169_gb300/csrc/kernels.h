@@ -27,6 +27,10 @@ cudaError_t launch_fg_rope(const int32_t* idx, int64_t n, int n_tensors, const v
                            int heads, int head_dim, bool bf16, int side, const int32_t axes[3], float theta,
                            int mode, int64_t T, int sms, cudaStream_t stream);
 
+// mask_alpha.cu
+cudaError_t launch_mask_from_alpha(const uint8_t* alpha, int n_views, int height, int width, int factor,
+                                   int radius, int threshold, uint8_t* canvas, cudaStream_t stream);
+
 // blockmask.cu
 struct MaskProblem {
   int64_t N;

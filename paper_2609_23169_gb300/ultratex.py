@@ -25,7 +25,7 @@ EXPORTS = (
     "ut_strerror", "ut_topk_count", "ut_fg_compact_workspace_size", "ut_fg_compact", "ut_fg_scatter",
     "ut_block_mask_workspace_size", "ut_block_mask", "ut_bsattn_fwd", "ut_bsattn_bwd_workspace_size",
     "ut_bsattn_bwd", "ut_fg_compact_noalloc", "ut_fg_euler_update", "ut_fg_composite",
-    "ut_fg_gather_rope", "ut_fg_scatter_rope",
+    "ut_fg_gather_rope", "ut_fg_scatter_rope", "ut_fg_mask_from_alpha",
 )
 
 
@@ -94,6 +94,8 @@ def lib() -> ctypes.CDLL:
     L.ut_fg_scatter_rope.restype = _i32
     L.ut_fg_scatter_rope.argtypes = [_vp, _i64, _i32, _ptrs, _ptrs, _i64, _i32, _i32, _i32, ctypes.POINTER(Rope),
                                      _i32, _vp]
+    L.ut_fg_mask_from_alpha.restype = _i32
+    L.ut_fg_mask_from_alpha.argtypes = [_vp, _i32, _i32, _i32, _i32, _i32, _i32, _vp, _vp]
     _lib = L
     return L
 
@@ -209,6 +211,23 @@ def ut_fg_scatter(idx: torch.Tensor, n: int, srcs: Sequence[torch.Tensor], dsts:
     st = lib().ut_fg_scatter(_p(idx), int(n), len(srcs), _ptr_array(srcs), _ptr_array(dsts), row_bytes, bg_mode,
                              _p(fill_row), T, _stream())
     _check("ut_fg_scatter", st)
+
+
+def ut_fg_mask_from_alpha(alpha: torch.Tensor, factor: int = 16, radius: int = 1, threshold: int = 0,
+                          out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Canvas mask [(2V + 1) * h * w] uint8 from alpha [V + 1, height, width] uint8 (views, then reference)."""
+    if alpha.dtype != torch.uint8 or alpha.dim() != 3 or not alpha.is_contiguous():
+        raise ValueError("alpha must be a contiguous [V + 1, height, width] uint8 tensor")
+    V = alpha.shape[0] - 1
+    H, W = alpha.shape[1], alpha.shape[2]
+    n = (2 * V + 1) * (H // max(factor, 1)) * (W // max(factor, 1))
+    if out is None:
+        out = torch.empty(max(n, 1), dtype=torch.uint8, device=alpha.device)
+    elif out.numel() < n or out.dtype != torch.uint8:
+        raise ValueError("out must hold (2V + 1) * (height/factor) * (width/factor) uint8")
+    st = lib().ut_fg_mask_from_alpha(_p(alpha), V, H, W, factor, radius, threshold, _p(out), _stream())
+    _check("ut_fg_mask_from_alpha", st)
+    return out[:n]
 
 
 def _rope_dims(ts: Sequence[torch.Tensor]):

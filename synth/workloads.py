@@ -17,7 +17,7 @@ order inside each image.
 
 Random streams (numpy PCG64 seeded with ``[seed, stream]``):
 mask=0, Q=1, K=2, V=3, dO=4, block fill=5, oracle row subsample=6, sampler
-latent=7, sampler velocity=8, background latent tile=9.
+latent=7, sampler velocity=8, background latent tile=9, alpha renders=10.
 Q/K/V/dO are drawn N(0,1) in fp32 and, for bf16 workloads, rounded to
 nearest-even bf16 by torch.
 """
@@ -31,7 +31,8 @@ import numpy as np
 import torch
 
 STREAM_MASK, STREAM_Q, STREAM_K, STREAM_V, STREAM_DO, STREAM_FILL, STREAM_ROWS = range(7)
-STREAM_LATENT, STREAM_VEL, STREAM_BG = 7, 8, 9
+STREAM_LATENT, STREAM_VEL, STREAM_BG, STREAM_ALPHA = 7, 8, 9, 10
+ALPHA_FACTOR = 16  # alpha pixels per token side (8x VAE downsampling, 2x2 patches)
 
 # Sampler-side latent: 16 VAE channels per 8x8 pixels, 2x2-patchified into one
 # token, i.e. 64 values per token; one step of a 28-step uniform schedule.
@@ -186,6 +187,34 @@ class Workload:
 
     def dout(self) -> torch.Tensor:
         return self._draw(STREAM_DO)
+
+    # -------------------------------------------------------- alpha renders
+    def alpha_images(self, factor: int = ALPHA_FACTOR) -> np.ndarray:
+        """[V + 1, side*factor, side*factor] uint8 alpha channels of the view
+        renders and the reference: a blob silhouette per image (sum of 3-6
+        Gaussians, thresholded so that ~0.45 fg_frac of the pixels are opaque; the pooling and dilation bring the token mask near fg_frac),
+        a two-pixel anti-aliased edge ramp, and sparse faint specks (alpha
+        1-20) in the background the way renders leave them."""
+        n_img = (N_VIEWS + 1) if self.multiview else self.n_images
+        P = self.side * factor
+        g = rng(self.seed, STREAM_ALPHA)
+        yy, xx = np.meshgrid((np.arange(P, dtype=np.float64) + 0.5) / factor,
+                             (np.arange(P, dtype=np.float64) + 0.5) / factor, indexing="ij")
+        out = np.zeros((n_img, P, P), dtype=np.uint8)
+        for i in range(n_img):
+            f = np.zeros_like(yy)
+            for _ in range(int(g.integers(3, 7))):
+                cy, cx = g.uniform(0.2, 0.8, size=2) * self.side
+                sig = g.uniform(0.08, 0.25) * self.side
+                f += g.uniform(0.5, 1.0) * np.exp(-((yy - cy) ** 2 + (xx - cx) ** 2) / (2.0 * sig * sig))
+            level = np.quantile(f, 1.0 - 0.45 * self.fg_frac)
+            band = 2.0 * float(np.abs(np.gradient(f)[0]).mean()) + 1e-12
+            a = np.clip((f - level) / band, 0.0, 1.0)
+            img = np.rint(a * 255.0).astype(np.uint8)
+            specks = g.random((P, P)) < 2e-4
+            img[specks & (img == 0)] = g.integers(1, 21, size=int((specks & (img == 0)).sum()), dtype=np.uint8)
+            out[i] = img
+        return out
 
     # ----------------------------------------------------- sampler inputs
     def sampler_inputs(self, channels: int = LATENT_CHANNELS, dtype: torch.dtype = torch.bfloat16) -> dict:

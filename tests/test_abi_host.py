@@ -144,6 +144,19 @@ def test_rope_argument_errors_are_caught_on_host(L):
     assert g(None, 0, 1, arr, arr, 10, 2, 128, u.UT_BF16, S(ok), None) == u.UT_OK                       # n = 0
 
 
+def test_alpha_mask_argument_errors_are_caught_on_host(L):
+    from paper_2609_23169_gb300 import ultratex as u
+    bogus = ctypes.c_void_p(16 * 1024)   # never dereferenced: every call must fail validation first
+    f = L.ut_fg_mask_from_alpha
+    assert f(bogus, 6, 2048, 2048, 0, 1, 0, bogus, None) == u.UT_ERR_INVALID_ARG       # factor 0
+    assert f(bogus, 6, 2040, 2048, 16, 1, 0, bogus, None) == u.UT_ERR_INVALID_ARG      # height not divisible
+    assert f(bogus, 6, 2048, 2048, 16, 17, 0, bogus, None) == u.UT_ERR_INVALID_ARG     # radius too large
+    assert f(bogus, 6, 2048, 2048, 16, 1, 256, bogus, None) == u.UT_ERR_INVALID_ARG    # threshold
+    assert f(bogus, -1, 2048, 2048, 16, 1, 0, bogus, None) == u.UT_ERR_INVALID_ARG     # views
+    assert f(None, 6, 2048, 2048, 16, 1, 0, bogus, None) == u.UT_ERR_INVALID_ARG       # no alpha
+    assert f(None, 6, 0, 2048, 16, 1, 0, None, None) == u.UT_OK                        # empty image
+
+
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     from paper_2609_23169_gb300 import ultratex as u
     monkeypatch.setattr(u, "_lib", None)
