@@ -131,6 +131,21 @@ def retained_flops(row_ptr, col_idx, N, b, d):
     return 4.0 * d * float((qsz * ksz).sum())
 
 
+def whole_job(ms_local: float, flops_local: float, world: int, device=None):
+    """Whole-job figures of a multi-rank run: the slowest rank's time (max over
+    ranks) and the work of all ranks (sum over ranks; replicas may process
+    different sequence lengths).  world == 1 returns the inputs."""
+    if world <= 1:
+        return float(ms_local), float(flops_local)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms_local)], dtype=torch.float64, device=device)
+    f = torch.tensor([float(flops_local)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(f, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(f.item())
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -211,12 +226,9 @@ def run_ours(args, rank, world, local_rank):
     kern_ms = {n: sum(a.elapsed_time(b) for a, b in l) / len(l) for n, l in ev.items()}
 
     # whole-job: max time over ranks, FLOPs summed over ranks (replicas)
-    if world > 1:
-        t = torch.tensor([ms_total], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total = float(t.item())
+    ms_total, flops_total = whole_job(ms_total, f_step * args.steps, world, dev)
     ms_step = ms_total / args.steps
-    value = world * f_step / (ms_step * 1e-3) / 1e12
+    value = flops_total / (ms_total * 1e-3) / 1e12
 
     # ---- e2e through host buffers: every step copies its canvas inputs from
     # pinned host memory and its canvas results back; three streams overlap
@@ -420,7 +432,7 @@ def time_rope(w, dev, hbm_peak: float, reps: int = 10) -> dict:
     idx = torch.from_numpy(np.flatnonzero(mask).astype(np.int32)).to(dev)
     N, T = int(idx.numel()), int(mask.size)
     q, k = w.q().to(dev), w.k().to(dev)
-    cfg = u.rope_config(w.side)
+    cfg = u.rope_config(w.side, prefix=w.text_prefix)
     qc, kc = (torch.empty((N, w.heads, w.head_dim), dtype=q.dtype, device=dev) for _ in range(2))
     dq, dk = torch.empty_like(q), torch.empty_like(k)
     row = w.heads * w.head_dim * q.element_size()

@@ -169,6 +169,9 @@ typedef struct {
   int32_t side;     /* tokens per image side */
   int32_t axes[3];  /* head dimensions of the image, y and x axes */
   float theta;      /* frequency base (10000) */
+  int32_t prefix;   /* text tokens before the images (0 or e.g. 512): canvas
+                       positions t < prefix are at (0, 0, 0), i.e. unrotated,
+                       and image coordinates count from t - prefix */
 } ut_rope;
 
 /* dst[n] = R(idx[n]) src[idx[n]] for n < n, every listed tensor (Q and K):

@@ -33,7 +33,9 @@ no blocking, fusion or reordering beyond what the definition states:
   head dimension is split into three axes (default 16/56/56 of 128); within
   axis a of d_a dimensions, pair k = (x[2k], x[2k+1]) is rotated by the angle
   pos_a * theta^(-2k/d_a) (theta = 10000).  Gathering Q and K applies the
-  rotation; scattering their gradients back applies its inverse.
+  rotation; scattering their gradients back applies its inverse.  Text tokens
+  placed before the images (the joint sequence's 512-token prefix of Table
+  S1) sit at position (0, 0, 0).
 * Sampler steps on the canvas latent: the sparse Euler update (Sec. 3.2,
   Eq. euler) moves only the retained positions by (t_prev - t_curr) times
   their predicted velocity; the composite latent (Sec. 3.4, Eq. mixed_latent)
@@ -127,12 +129,19 @@ def canvas_mask_from_alpha(alpha: np.ndarray, factor: int = 16, radius: int = 1,
 
 
 # --------------------------------------------------------------------- RoPE
-def rope_positions(idx: np.ndarray, side: int) -> np.ndarray:
+def rope_positions(idx: np.ndarray, side: int, prefix: int = 0) -> np.ndarray:
     """Canvas positions -> (image, y, x) of images of side x side tokens, stored
-    one after another in raster order.  [n] -> [n, 3] int64."""
+    one after another in raster order.  [n] -> [n, 3] int64.
+
+    With a text prefix (the joint sequence of the MM-DiT carries its text
+    tokens before the images), positions t < prefix are text tokens at
+    (0, 0, 0) and image coordinates count from t - prefix."""
     t = np.asarray(idx, dtype=np.int64)
     s2 = int(side) * int(side)
-    return np.stack([t // s2, (t % s2) // side, t % side], axis=1)
+    ti = t - int(prefix)
+    pos = np.stack([ti // s2, (ti % s2) // side, ti % side], axis=1)
+    pos[t < int(prefix)] = 0
+    return pos
 
 
 def rope_angles(pos: np.ndarray, head_dim: int, axes=(16, 56, 56), theta: float = 10000.0) -> np.ndarray:
@@ -166,19 +175,20 @@ def rope_rotate(x: np.ndarray, angles: np.ndarray, inverse: bool = False) -> np.
     return y
 
 
-def fg_compact_rope(mask: np.ndarray, x: np.ndarray, side: int, axes=(16, 56, 56), theta: float = 10000.0):
+def fg_compact_rope(mask: np.ndarray, x: np.ndarray, side: int, axes=(16, 56, 56), theta: float = 10000.0,
+                    prefix: int = 0):
     """Gather of Q or K (Sec. 3.2) with the rotary embedding of each retained
     token's original canvas position applied.  Returns (idx, rotated rows)."""
     idx, (xc,) = fg_compact(mask, [x])
-    ang = rope_angles(rope_positions(idx, side), np.asarray(x).shape[-1], axes, theta)
+    ang = rope_angles(rope_positions(idx, side, prefix), np.asarray(x).shape[-1], axes, theta)
     return idx, rope_rotate(xc, ang)
 
 
 def fg_scatter_rope(idx: np.ndarray, src: np.ndarray, dst_in: np.ndarray, side: int, mode: int = BG_ZERO,
-                    axes=(16, 56, 56), theta: float = 10000.0) -> np.ndarray:
+                    axes=(16, 56, 56), theta: float = 10000.0, prefix: int = 0) -> np.ndarray:
     """Scatter of dQ or dK back to the canvas through the inverse rotation (the
     gradient of the rotated gather); background rows per ``mode``."""
-    ang = rope_angles(rope_positions(idx, side), np.asarray(src).shape[-1], axes, theta)
+    ang = rope_angles(rope_positions(idx, side, prefix), np.asarray(src).shape[-1], axes, theta)
     return fg_scatter(idx, rope_rotate(src, ang, inverse=True), dst_in, mode)
 
 

@@ -174,7 +174,8 @@ static ut_status check_rope(int64_t n, int64_t T, int32_t n_tensors, const void*
                             bool gather) {
   if (n < 0 || T < 0 || n > T || n_tensors < 1 || n_tensors > 8 || heads < 1 || head_dim < 2) return UT_ERR_INVALID_ARG;
   if (dtype != UT_BF16 && dtype != UT_F32) return UT_ERR_INVALID_ARG;
-  if (!rope || !h_src || !h_dst || rope->side < 1 || !(rope->theta > 0.0f) || !isfinite(rope->theta))
+  if (!rope || !h_src || !h_dst || rope->side < 1 || rope->prefix < 0 || !(rope->theta > 0.0f) ||
+      !isfinite(rope->theta))
     return UT_ERR_INVALID_ARG;
   if (rope->axes[0] < 0 || rope->axes[1] < 0 || rope->axes[2] < 0 || rope->axes[0] % 2 || rope->axes[1] % 2 ||
       rope->axes[2] % 2 || (int64_t)rope->axes[0] + rope->axes[1] + rope->axes[2] != head_dim)
@@ -198,7 +199,7 @@ ut_status ut_fg_gather_rope(const int32_t* idx, int64_t n, int32_t n_tensors, co
   if (n == 0) return UT_OK;
   if (!idx) return UT_ERR_INVALID_ARG;
   return from_cuda(launch_fg_rope(idx, n, n_tensors, h_src, h_dst, heads, head_dim, dtype == UT_BF16, rope->side,
-                                  rope->axes, rope->theta, 0, T, device_sms(), static_cast<cudaStream_t>(stream)));
+                                  rope->prefix, rope->axes, rope->theta, 0, T, device_sms(), static_cast<cudaStream_t>(stream)));
 }
 
 ut_status ut_fg_scatter_rope(const int32_t* idx, int64_t n, int32_t n_tensors, const void* const* h_src,
@@ -211,7 +212,7 @@ ut_status ut_fg_scatter_rope(const int32_t* idx, int64_t n, int32_t n_tensors, c
   const int mode = bg_mode == UT_BG_KEEP ? 1 : 2;
   if ((mode == 1 && n == 0) || T == 0) return UT_OK;
   return from_cuda(launch_fg_rope(idx, n, n_tensors, h_src, h_dst, heads, head_dim, dtype == UT_BF16, rope->side,
-                                  rope->axes, rope->theta, mode, T, device_sms(), static_cast<cudaStream_t>(stream)));
+                                  rope->prefix, rope->axes, rope->theta, mode, T, device_sms(), static_cast<cudaStream_t>(stream)));
 }
 
 ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int32_t channels,

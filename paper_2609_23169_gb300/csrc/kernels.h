@@ -24,8 +24,8 @@ cudaError_t launch_fg_composite(const uint8_t* mask, int64_t T, void* z, const v
 
 // rope.cu (mode: 0 gather, 1 scatter keeping the background, 2 scatter zeroing it)
 cudaError_t launch_fg_rope(const int32_t* idx, int64_t n, int n_tensors, const void* const* src, void* const* dst,
-                           int heads, int head_dim, bool bf16, int side, const int32_t axes[3], float theta,
-                           int mode, int64_t T, int sms, cudaStream_t stream);
+                           int heads, int head_dim, bool bf16, int side, int prefix, const int32_t axes[3],
+                           float theta, int mode, int64_t T, int sms, cudaStream_t stream);
 
 // mask_alpha.cu
 cudaError_t launch_mask_from_alpha(const uint8_t* alpha, int n_views, int height, int width, int factor,

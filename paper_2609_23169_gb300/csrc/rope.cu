@@ -2,8 +2,9 @@
 // gradient scatter (Sec. 3.2: every retained token keeps its original RoPE
 // index, i.e. its canvas position).
 //
-//   canvas position t of images of side S (one after another, raster order)
-//     -> (image, y, x) = (t / S^2, (t mod S^2) / S, t mod S);
+//   canvas position t of images of side S (one after another, raster order,
+//   after `prefix` text tokens that stay unrotated)
+//     -> (image, y, x) = (t' / S^2, (t' mod S^2) / S, t' mod S), t' = t - prefix;
 //   head dimension split into three axes; pair p = (x[2p], x[2p+1]) belongs
 //   to axis a(p) and turns by pos_a * freq[p], freq = theta^(-2k/d_a) for the
 //   k-th pair of its axis (table computed on the host in double precision).
@@ -38,7 +39,8 @@ struct RopeParams {
 template <bool kBf16, int kMode, int kVec>
 __global__ void __launch_bounds__(kRopeThreads) rope_kernel(const __grid_constant__ RopeParams prm, int n_tensors,
                                                              const int32_t* __restrict__ idx, int64_t n, int64_t T,
-                                                             int side, int64_t row_bytes, int vec_per_head) {
+                                                             int side, int prefix, int64_t row_bytes,
+                                                             int vec_per_head) {
   constexpr int kPairs = kBf16 ? 4 : 2;  // pairs per 16-byte vector
   constexpr bool kInverse = kMode != kGather;
   const int lane = threadIdx.x & 31;
@@ -76,7 +78,9 @@ __global__ void __launch_bounds__(kRopeThreads) rope_kernel(const __grid_constan
           w[j] = (r >= 0 && v < nvec) ? ld_nc_v4(s + (v << 4)) : make_uint4(0, 0, 0, 0);
         }
         if (ti == 0 && v0 == 0 && r >= 0) {  // this lane's pairs, once per row, while the loads fly
-          const float pi = (float)(t / s2), py = (float)((t % s2) / side), px = (float)(t % side);
+          const int64_t ti = t - prefix;  // text tokens (t < prefix) sit at (0, 0, 0)
+          const float pi = ti < 0 ? 0.f : (float)(ti / s2), py = ti < 0 ? 0.f : (float)((ti % s2) / side);
+          const float px = ti < 0 ? 0.f : (float)(ti % side);
 #pragma unroll
           for (int e = 0; e < kPairs; ++e) {
             const int p = p0 + e;
@@ -114,8 +118,8 @@ __global__ void __launch_bounds__(kRopeThreads) rope_kernel(const __grid_constan
 }
 
 cudaError_t launch_fg_rope(const int32_t* idx, int64_t n, int n_tensors, const void* const* src, void* const* dst,
-                           int heads, int head_dim, bool bf16, int side, const int32_t axes[3], float theta,
-                           int mode, int64_t T, int sms, cudaStream_t stream) {
+                           int heads, int head_dim, bool bf16, int side, int prefix, const int32_t axes[3],
+                           float theta, int mode, int64_t T, int sms, cudaStream_t stream) {
   RopeParams prm{};
   for (int i = 0; i < n_tensors; ++i) {
     prm.src[i] = static_cast<const uint8_t*>(src[i]);
@@ -136,10 +140,10 @@ cudaError_t launch_fg_rope(const int32_t* idx, int64_t n, int n_tensors, const v
   const int grid = (int)(want < cap ? want : cap);
   const bool big = row_bytes >= 16 * 32 * 12;
 #define UT_ROPE_LAUNCH(B, M)                                                                                       \
-  (big ? rope_kernel<B, M, 12><<<grid, kRopeThreads, 0, stream>>>(prm, n_tensors, idx, n, T, side, row_bytes,    \
-                                                                  vec_per_head)                                  \
-       : rope_kernel<B, M, 4><<<grid, kRopeThreads, 0, stream>>>(prm, n_tensors, idx, n, T, side, row_bytes,     \
-                                                                 vec_per_head))
+  (big ? rope_kernel<B, M, 12><<<grid, kRopeThreads, 0, stream>>>(prm, n_tensors, idx, n, T, side, prefix,       \
+                                                                  row_bytes, vec_per_head)                                  \
+       : rope_kernel<B, M, 4><<<grid, kRopeThreads, 0, stream>>>(prm, n_tensors, idx, n, T, side, prefix,        \
+                                                                 row_bytes, vec_per_head))
   if (bf16) {
     if (mode == kGather) UT_ROPE_LAUNCH(true, kGather);
     else if (mode == kScatterKeep) UT_ROPE_LAUNCH(true, kScatterKeep);

@@ -41,12 +41,13 @@ class AttnShape(ctypes.Structure):
 
 
 class Rope(ctypes.Structure):
-    """ut_rope: tokens per image side, head dimensions of the image / y / x axes, frequency base."""
-    _fields_ = [("side", ctypes.c_int32), ("axes", ctypes.c_int32 * 3), ("theta", ctypes.c_float)]
+    """ut_rope: tokens per image side, head dimensions of the image / y / x axes, frequency base, text prefix."""
+    _fields_ = [("side", ctypes.c_int32), ("axes", ctypes.c_int32 * 3), ("theta", ctypes.c_float),
+                ("prefix", ctypes.c_int32)]
 
 
-def rope_config(side: int, axes=(16, 56, 56), theta: float = 10000.0) -> Rope:
-    return Rope(int(side), (ctypes.c_int32 * 3)(*axes), float(theta))
+def rope_config(side: int, axes=(16, 56, 56), theta: float = 10000.0, prefix: int = 0) -> Rope:
+    return Rope(int(side), (ctypes.c_int32 * 3)(*axes), float(theta), int(prefix))
 
 
 _lib = None

@@ -67,6 +67,7 @@ class Workload:
     density: float         # structured: target density (random fill up to it); topk: rho
     tiny_fill: Optional[float] = None  # tiny case: fixed fill probability of non-own tiles
     seed: int = 0
+    text_prefix: int = 0   # text tokens of the joint MM-DiT sequence before the images (always kept)
 
     # ---------------------------------------------------------------- sizes
     @property
@@ -79,7 +80,7 @@ class Workload:
 
     @property
     def T(self) -> int:
-        return self.n_images * self.tokens_per_image
+        return self.text_prefix + self.n_images * self.tokens_per_image
 
     def image_counts(self) -> np.ndarray:
         """Foreground tokens per image (exact counts, round half up)."""
@@ -91,7 +92,7 @@ class Workload:
 
     @property
     def N(self) -> int:
-        return int(self.image_counts().sum())
+        return self.text_prefix + int(self.image_counts().sum())
 
     @property
     def n_tiles(self) -> int:
@@ -159,7 +160,11 @@ class Workload:
         return masks
 
     def canvas_mask(self) -> np.ndarray:
-        return np.ascontiguousarray(self.image_masks().reshape(-1))
+        """[T] uint8: the text prefix (always kept), then the images one after another."""
+        m = self.image_masks().reshape(-1)
+        if self.text_prefix:
+            m = np.concatenate([np.ones(self.text_prefix, np.uint8), m])
+        return np.ascontiguousarray(m)
 
     # --------------------------------------------------------------- tensors
     def _draw(self, stream: int, rows: Optional[int] = None) -> torch.Tensor:
@@ -225,7 +230,7 @@ class Workload:
         canonical background latent tile, and the step dt = t_prev - t_curr."""
         n_img = N_VIEWS if self.multiview else self.n_images
         T = n_img * self.tokens_per_image
-        mask = self.canvas_mask()[:T].copy()
+        mask = self.canvas_mask()[self.text_prefix:self.text_prefix + T].copy()
         n = int(mask.sum())
         z = rng(self.seed, STREAM_LATENT).standard_normal((T, channels), dtype=np.float32)
         v = rng(self.seed, STREAM_VEL).standard_normal((n, channels), dtype=np.float32)
@@ -243,6 +248,7 @@ class Workload:
         Compacted rows keep canvas order, so image boundaries in compacted
         order are the running sums of the per-image foreground counts.
         """
+        assert self.text_prefix == 0, "the structured rule is defined for image tokens only"
         bounds = np.concatenate([[0], np.cumsum(self.image_counts())])
         out = []
         for i in range(self.n_tiles):
@@ -319,6 +325,11 @@ CONFIGS: dict[str, Workload] = {
     "c2048": Workload("c2048", n_images=13, side=128, fg_frac=0.40, shape="blob", ref_full=False,
                       heads=24, head_dim=128, dtype="bf16", block=128, mask_mode="topk",
                       density=0.12),
+    # the 2048 canvas with the joint sequence's 512 text tokens in front (the
+    # token lengths of Table S1 include them): T = 213,504, N = 85,714
+    "c2048t": Workload("c2048t", n_images=13, side=128, fg_frac=0.40, shape="blob", ref_full=False,
+                       heads=24, head_dim=128, dtype="bf16", block=128, mask_mode="topk",
+                       density=0.12, text_prefix=512),
 }
 
 SWEEP_FG = (0.20, 0.40, 0.60, 0.80)

@@ -437,6 +437,13 @@ def check_rope(o):
     back = o.fg_scatter_rope(idx, xr, np.zeros_like(xt), side, o.BG_ZERO)
     if not (np.allclose(back[idx], xt[idx], atol=1e-12) and not back[m == 0].any()):
         bad.append("rope scatter is not the inverse of the rope gather")
+    # a text prefix: its tokens are not rotated, image tokens keep the
+    # coordinates they have without the prefix
+    pre = 7
+    tp = np.concatenate([np.arange(pre), pre + idx]).astype(np.int64)
+    pp = o.rope_positions(tp, side, prefix=pre)
+    if pp[:pre].any() or not np.array_equal(pp[pre:], o.rope_positions(idx, side)):
+        bad.append("text prefix positions")
     return bad
 
 

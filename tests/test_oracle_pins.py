@@ -235,9 +235,15 @@ def _rope_freq_k_over_d(pos, head_dim, axes=(16, 56, 56), theta=10000.0):
     return np.concatenate(cols, axis=1)
 
 
-def _rope_xy_swapped(idx, side):
-    p = o.rope_positions(idx, side)
+def _rope_xy_swapped(idx, side, prefix=0):
+    p = o.rope_positions(idx, side, prefix)
     return p[:, [0, 2, 1]]
+
+
+def _rope_prefix_rotated(idx, side, prefix=0):
+    t = np.asarray(idx, dtype=np.int64) - prefix   # text tokens treated as images at negative positions
+    s2 = side * side
+    return np.stack([t // s2, (t % s2) // side, t % side], axis=1)
 
 
 def _alpha_all_pixels(alpha, factor=16, radius=1, threshold=0):
@@ -298,6 +304,7 @@ def _csr_descending(bm):
     ("RoPE pairing halves instead of neighbours", lambda: pins.check_rope(_OracleWith(rope_rotate=_rope_half_split))),
     ("RoPE frequencies theta^(-k/d)", lambda: pins.check_rope(_OracleWith(rope_angles=_rope_freq_k_over_d))),
     ("RoPE with x and y swapped", lambda: pins.check_rope(_OracleWith(rope_positions=_rope_xy_swapped))),
+    ("RoPE rotating the text prefix", lambda: pins.check_rope(_OracleWith(rope_positions=_rope_prefix_rotated))),
     ("Euler step with t_curr - t_prev", lambda: pins.check_sampler(_euler_sign_flipped, o.fg_composite, o.fg_scatter)),
     ("Euler step on rows 0..n-1", lambda: pins.check_sampler(_euler_rows_in_order, o.fg_composite, o.fg_scatter)),
     ("composite tile indexed by t // P", lambda: pins.check_sampler(o.fg_euler_update, _composite_tile_by_block,
