@@ -10,7 +10,8 @@ no blocking, fusion or reordering beyond what the definition states:
 * Background Token Dropping (Sec. 3.2): ``z~ = Gather_{M_fg}(z)``; each
   retained token keeps its canvas position (its RoPE index).
 * Block partition (Sec. 3.3): Q into query blocks of b_q rows, K/V into key
-  blocks of b_kv rows.
+  blocks of b_kv rows (the functions take b = b_q and an optional b_kv,
+  equal to b when not given).
 * Compressed scores and Top-K (Sec. 3.3, the equation for S_c and the one
   for M_c): ``S_c = pool(Q) pool(K)^T`` with mean pooling per block, and per
   head and query block the K_rho = floor(rho * N_k) key blocks of largest score.
@@ -279,27 +280,31 @@ def k_rho(rho: float, nk: int) -> int:
     return max(1, int(math.floor(float(rho) * int(nk))))
 
 
-def compressed_scores(qc_h: np.ndarray, kc_h: np.ndarray, b: int) -> np.ndarray:
-    """S_c = pool(Q) pool(K)^T for one head (Sec. 3.3)."""
-    return block_pool(qc_h, b) @ block_pool(kc_h, b).T
+def compressed_scores(qc_h: np.ndarray, kc_h: np.ndarray, b: int, b_kv: Optional[int] = None) -> np.ndarray:
+    """S_c = pool(Q) pool(K)^T for one head (Sec. 3.3); Q pooled over b_q = b rows,
+    K over b_kv rows (b_kv = b when not given)."""
+    return block_pool(qc_h, b) @ block_pool(kc_h, b if b_kv is None else b_kv).T
 
 
-def topk_block_mask(qc: np.ndarray, kc: np.ndarray, b: int, rho: float):
+def topk_block_mask(qc: np.ndarray, kc: np.ndarray, b: int, rho: float, b_kv: Optional[int] = None):
     """Per head and query block, the K_rho key blocks with the largest S_c (Sec. 3.3).
 
-    qc, kc: [N, H, d].  Returns (row_ptr, col_idx, scores [H, N_q, N_k], K_rho);
-    lists ascending, ties toward the smaller key-block index.
+    qc, kc: [N, H, d]; query blocks of b rows, key blocks of b_kv rows (b when
+    not given), K_rho = max(1, floor(rho N_k)).  Returns (row_ptr, col_idx,
+    scores [H, N_q, N_k], K_rho); lists ascending, ties toward the smaller
+    key-block index.
     """
     N, H, _ = qc.shape
-    nq = n_blocks(N, b)
-    kr = k_rho(rho, nq)
-    scores = np.zeros((H, nq, nq))
+    bk = b if b_kv is None else b_kv
+    nq, nk = n_blocks(N, b), n_blocks(N, bk)
+    kr = k_rho(rho, nk)
+    scores = np.zeros((H, nq, nk))
     lists = []
     for h in range(H):
-        sc = compressed_scores(qc[:, h], kc[:, h], b)
+        sc = compressed_scores(qc[:, h], kc[:, h], b, bk)
         scores[h] = sc
         for i in range(nq):
-            order = np.lexsort((np.arange(nq), -sc[i]))   # score desc, index asc
+            order = np.lexsort((np.arange(nk), -sc[i]))   # score desc, index asc
             lists.append(np.sort(order[:kr]))
     row_ptr = np.arange(H * nq + 1, dtype=np.int64) * kr
     col_idx = np.concatenate(lists) if lists else np.zeros(0, np.int64)
@@ -326,21 +331,23 @@ def _row_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float):
     return p @ v, (m + np.log(l))[:, 0], p
 
 
-def bsattn_fwd(qc, kc, vc, row_ptr, col_idx, b: int, scale: Optional[float] = None):
+def bsattn_fwd(qc, kc, vc, row_ptr, col_idx, b: int, scale: Optional[float] = None, b_kv: Optional[int] = None):
     """Block-sparse attention forward (Sec. 3.3): O_i = softmax(Q_i K_{S_i}^T/sqrt d) V_{S_i}.
 
-    qc, kc, vc: [N, H, d].  Returns O [N, H, d] and LSE [H, N] (natural log).
+    qc, kc, vc: [N, H, d]; query blocks of b rows, key blocks of b_kv rows (b
+    when not given).  Returns O [N, H, d] and LSE [H, N] (natural log).
     """
     qc, kc, vc = (np.asarray(a, dtype=np.float64) for a in (qc, kc, vc))
     N, H, d = qc.shape
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    bk = b if b_kv is None else b_kv
     nq = n_blocks(N, b)
     O = np.zeros((N, H, d))
     LSE = np.full((H, N), -np.inf)
     for h in range(H):
         for i in range(nq):
             rows = tile_rows(i, N, b)
-            keys = _keys(row_ptr, col_idx, h * nq + i, N, b)
+            keys = _keys(row_ptr, col_idx, h * nq + i, N, bk)
             o, lse, _ = _row_attention(qc[rows, h], kc[keys, h], vc[keys, h], scale)
             O[rows, h] = o
             LSE[h, rows] = lse
@@ -348,17 +355,18 @@ def bsattn_fwd(qc, kc, vc, row_ptr, col_idx, b: int, scale: Optional[float] = No
 
 
 def bsattn_fwd_rows(qc, kc, vc, row_ptr, col_idx, b: int, h: int, rows: np.ndarray,
-                    scale: Optional[float] = None):
+                    scale: Optional[float] = None, b_kv: Optional[int] = None):
     """The forward for a subset of query rows of head h (spot checks at full size)."""
     N, H, d = qc.shape
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    bk = b if b_kv is None else b_kv
     nq = n_blocks(N, b)
     rows = np.asarray(rows, dtype=np.int64)
     O = np.zeros((len(rows), d))
     LSE = np.full(len(rows), -np.inf)
     for t in np.unique(rows // b):
         sel = np.flatnonzero(rows // b == t)
-        keys = _keys(row_ptr, col_idx, h * nq + int(t), N, b)
+        keys = _keys(row_ptr, col_idx, h * nq + int(t), N, bk)
         q = np.asarray(qc[rows[sel], h], dtype=np.float64)
         o, lse, _ = _row_attention(q, np.asarray(kc[keys, h], np.float64),
                                    np.asarray(vc[keys, h], np.float64), scale)
@@ -368,7 +376,8 @@ def bsattn_fwd_rows(qc, kc, vc, row_ptr, col_idx, b: int, h: int, rows: np.ndarr
 
 
 # ----------------------------------------------------- attention backward
-def bsattn_bwd(qc, kc, vc, dout, row_ptr, col_idx, b: int, scale: Optional[float] = None):
+def bsattn_bwd(qc, kc, vc, dout, row_ptr, col_idx, b: int, scale: Optional[float] = None,
+               b_kv: Optional[int] = None):
     """Gradients of the block-sparse forward w.r.t. Q, K, V.
 
     Per retained (query row r, key row k): P = softmax row, D_r = dO_r . O_r,
@@ -378,6 +387,7 @@ def bsattn_bwd(qc, kc, vc, dout, row_ptr, col_idx, b: int, scale: Optional[float
     qc, kc, vc, dout = (np.asarray(a, dtype=np.float64) for a in (qc, kc, vc, dout))
     N, H, d = qc.shape
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    bk = b if b_kv is None else b_kv
     nq = n_blocks(N, b)
     dQ = np.zeros_like(qc)
     dK = np.zeros_like(kc)
@@ -385,7 +395,7 @@ def bsattn_bwd(qc, kc, vc, dout, row_ptr, col_idx, b: int, scale: Optional[float
     for h in range(H):
         for i in range(nq):
             rows = tile_rows(i, N, b)
-            keys = _keys(row_ptr, col_idx, h * nq + i, N, b)
+            keys = _keys(row_ptr, col_idx, h * nq + i, N, bk)
             if len(keys) == 0:
                 continue
             q, k, v, do = qc[rows, h], kc[keys, h], vc[keys, h], dout[rows, h]
@@ -400,16 +410,17 @@ def bsattn_bwd(qc, kc, vc, dout, row_ptr, col_idx, b: int, scale: Optional[float
 
 
 def bsattn_bwd_dq_rows(qc, kc, vc, dout, row_ptr, col_idx, b: int, h: int, rows: np.ndarray,
-                       scale: Optional[float] = None):
+                       scale: Optional[float] = None, b_kv: Optional[int] = None):
     """dQ for a subset of query rows of head h."""
     N, H, d = qc.shape
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    bk = b if b_kv is None else b_kv
     nq = n_blocks(N, b)
     rows = np.asarray(rows, dtype=np.int64)
     dQ = np.zeros((len(rows), d))
     for t in np.unique(rows // b):
         sel = np.flatnonzero(rows // b == t)
-        keys = _keys(row_ptr, col_idx, h * nq + int(t), N, b)
+        keys = _keys(row_ptr, col_idx, h * nq + int(t), N, bk)
         if len(keys) == 0:
             continue
         q = np.asarray(qc[rows[sel], h], np.float64)
@@ -423,7 +434,7 @@ def bsattn_bwd_dq_rows(qc, kc, vc, dout, row_ptr, col_idx, b: int, h: int, rows:
 
 
 def bsattn_bwd_dkdv_rows(qc, kc, vc, dout, row_ptr, col_idx, b: int, h: int,
-                         key_rows: np.ndarray, scale: Optional[float] = None):
+                         key_rows: np.ndarray, scale: Optional[float] = None, b_kv: Optional[int] = None):
     """dK, dV for a subset of key rows of head h.
 
     A key row in block j gathers contributions from every query block i whose
@@ -432,11 +443,12 @@ def bsattn_bwd_dkdv_rows(qc, kc, vc, dout, row_ptr, col_idx, b: int, h: int,
     """
     N, H, d = qc.shape
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    bk = b if b_kv is None else b_kv
     nq = n_blocks(N, b)
     key_rows = np.asarray(key_rows, dtype=np.int64)
     dK = np.zeros((len(key_rows), d))
     dV = np.zeros((len(key_rows), d))
-    want = set(int(x) // b for x in key_rows)
+    want = set(int(x) // bk for x in key_rows)
     for i in range(nq):
         r = h * nq + i
         tiles = set(int(x) for x in col_idx[row_ptr[r]:row_ptr[r + 1]])
@@ -444,7 +456,7 @@ def bsattn_bwd_dkdv_rows(qc, kc, vc, dout, row_ptr, col_idx, b: int, h: int,
         if not hit:
             continue
         rows = tile_rows(i, N, b)
-        keys = _keys(row_ptr, col_idx, r, N, b)
+        keys = _keys(row_ptr, col_idx, r, N, bk)
         q = np.asarray(qc[rows, h], np.float64)
         k = np.asarray(kc[keys, h], np.float64)
         v = np.asarray(vc[keys, h], np.float64)
@@ -463,12 +475,14 @@ def bsattn_bwd_dkdv_rows(qc, kc, vc, dout, row_ptr, col_idx, b: int, h: int,
 
 
 # ------------------------------------------------------------------ FLOPs
-def retained_flops_fwd(row_ptr, col_idx, n: int, b: int, d: int) -> float:
+def retained_flops_fwd(row_ptr, col_idx, n: int, b: int, d: int, b_kv: Optional[int] = None) -> float:
     """4 * |Q_i| * |K_j| * d per retained (head, i, j) pair, actual tail sizes."""
-    nq = n_blocks(n, b)
-    sizes = np.array([len(tile_rows(j, n, b)) for j in range(nq)], dtype=np.float64)
+    bk = b if b_kv is None else b_kv
+    nq, nk = n_blocks(n, b), n_blocks(n, bk)
+    qs = np.array([len(tile_rows(i, n, b)) for i in range(nq)], dtype=np.float64)
+    ks = np.array([len(tile_rows(j, n, bk)) for j in range(nk)], dtype=np.float64)
     total = 0.0
     for r in range(len(row_ptr) - 1):
         i = r % nq
-        total += sizes[i] * sizes[col_idx[row_ptr[r]:row_ptr[r + 1]]].sum()
+        total += qs[i] * ks[col_idx[row_ptr[r]:row_ptr[r + 1]]].sum()
     return 4.0 * d * total

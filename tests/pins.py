@@ -500,3 +500,55 @@ def check_alpha_mask(token_mask_from_alpha, canvas_mask_from_alpha):
         if not np.array_equal(blocks[2 * V], token_mask_from_alpha(stack[V], f, 1, 0).ravel()):
             bad.append("reference mask")
     return bad
+
+
+# --------------------------------------------------- unequal block sizes
+def check_unequal_blocks(o):
+    """Query blocks of b_q rows and key blocks of b_kv rows (Sec. 3.3 defines
+    both sizes): Top-K by brute force, forward and backward against masked
+    SDPA, FLOPs against the expanded token mask."""
+    bad = []
+    g = np.random.Generator(np.random.PCG64(29))
+    for N, H, d, bq, bk in ((23, 2, 6, 4, 2), (23, 2, 6, 2, 5), (16, 1, 4, 8, 4)):
+        q, k, v, do = (g.standard_normal((N, H, d)) for _ in range(4))
+        nq, nk = -(-N // bq), -(-N // bk)
+        # Top-K over N_k key blocks of b_kv rows
+        for rho in (0.2, 0.5):
+            rp, ci, _, kr = o.topk_block_mask(q, k, bq, rho, b_kv=bk)
+            if kr != max(1, math.floor(rho * nk)) or len(rp) != H * nq + 1:
+                bad.append(f"K_rho / list count for b_q={bq}, b_kv={bk}")
+                continue
+            for h in range(H):
+                mq = [q[i * bq:min(N, i * bq + bq), h].mean(0) for i in range(nq)]
+                mk = [k[j * bk:min(N, j * bk + bk), h].mean(0) for j in range(nk)]
+                for i in range(nq):
+                    s = [float(np.dot(mq[i], mk[j])) for j in range(nk)]
+                    want = sorted(sorted(range(nk), key=lambda j: (-s[j], j))[:kr])
+                    r = h * nq + i
+                    if list(ci[rp[r]:rp[r + 1]]) != want:
+                        bad.append(f"brute-force Top-K b_q={bq} b_kv={bk} rho={rho}")
+                        break
+        # forward / backward against SDPA with the token mask bm[h, r // b_q, c // b_kv]
+        bm = (g.random((H, nq, nk)) < 0.5).astype(np.uint8)
+        for h in range(H):
+            for i in range(nq):
+                if not bm[h, i].any():
+                    bm[h, i, g.integers(nk)] = 1
+        rp, ci = o.bitmap_to_csr(bm)
+        tm = np.zeros((H, N, N), dtype=bool)
+        for h in range(H):
+            for r in range(N):
+                for c in range(N):
+                    tm[h, r, c] = bool(bm[h, r // bq, c // bk])
+        scale = 1.0 / math.sqrt(d)
+        O, _ = o.bsattn_fwd(q, k, v, rp, ci, bq, b_kv=bk)
+        _, gq, gk, gv = sdpa_reference(q, k, v, tm, scale, True, do)
+        if not _close(O, sdpa_reference(q, k, v, tm, scale), 1e-10):
+            bad.append(f"forward b_q={bq} b_kv={bk} != masked SDPA")
+        dQ, dK, dV = o.bsattn_bwd(q, k, v, do, rp, ci, bq, b_kv=bk)
+        for name, a, r_ in (("dQ", dQ, gq), ("dK", dK, gk), ("dV", dV, gv)):
+            if not _close(a, r_, 1e-9):
+                bad.append(f"{name} b_q={bq} b_kv={bk} != autograd")
+        if not np.isclose(o.retained_flops_fwd(rp, ci, N, bq, d, b_kv=bk), 4.0 * d * tm.sum()):
+            bad.append(f"FLOPs b_q={bq} b_kv={bk}")
+    return bad

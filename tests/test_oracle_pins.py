@@ -35,6 +35,10 @@ def test_sampler_steps_pinned():
     assert pins.check_sampler(o.fg_euler_update, o.fg_composite, o.fg_scatter) == []
 
 
+def test_unequal_blocks_pinned():
+    assert pins.check_unequal_blocks(o) == []
+
+
 def test_alpha_mask_pinned():
     assert pins.check_alpha_mask(o.token_mask_from_alpha, o.canvas_mask_from_alpha) == []
 
@@ -269,6 +273,14 @@ def _canvas_conditions_use_reference(alpha, factor=16, radius=1, threshold=0):
     return np.concatenate(views + [ref] * V + [ref]).astype(np.uint8)
 
 
+def _fwd_keys_at_query_size(q, k, v, rp, ci, b, scale=None, b_kv=None):
+    return o.bsattn_fwd(q, k, v, rp, ci, b, scale)
+
+
+def _topk_pool_k_at_query_size(qc, kc, b, rho, b_kv=None):
+    return o.topk_block_mask(qc, kc, b, rho)
+
+
 def _csr_descending(bm):
     rp, ci = o.bitmap_to_csr(bm)
     ci = ci.copy()
@@ -292,6 +304,8 @@ def _csr_descending(bm):
     ("compaction off by one", lambda: pins.check_compaction(_compact_off_by_one, o.fg_scatter)),
     ("scatter ignores the mode", lambda: pins.check_compaction(o.fg_compact, _scatter_zero_everything)),
     ("CSR lists descending", lambda: pins.check_block_lists(_csr_descending, o.csr_to_csc)),
+    ("b_kv ignored by the forward", lambda: pins.check_unequal_blocks(_OracleWith(bsattn_fwd=_fwd_keys_at_query_size))),
+    ("b_kv ignored by Top-K", lambda: pins.check_unequal_blocks(_OracleWith(topk_block_mask=_topk_pool_k_at_query_size))),
     ("alpha pooled with all() instead of any()", lambda: pins.check_alpha_mask(_alpha_all_pixels,
                                                                                o.canvas_mask_from_alpha)),
     ("alpha dilation one token too wide", lambda: pins.check_alpha_mask(_alpha_radius_plus_one,
