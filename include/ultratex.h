@@ -60,17 +60,22 @@ enum { UT_BG_KEEP = 0, UT_BG_ZERO = 1, UT_BG_FILL = 2 };
 enum { UT_MASK_TOPK = 0, UT_MASK_BITMAP = 1 };
 
 /* Shape of the compacted attention problem.  Sec. 3.3 states it per head as
- * Q, K, V in R^{N x d} partitioned into blocks of b_q and b_kv rows; here
- * b_q = b_kv = block.  N_q = N_k = ceil(N / block); the last block may be
- * partial (its missing key rows are excluded, its missing query rows are not
- * written). */
+ * Q, K, V in R^{N x d} partitioned into query blocks of b_q = block rows and
+ * key blocks of b_kv = block_k rows (block_k = 0: b_kv = b_q).
+ * N_q = ceil(N / b_q), N_k = ceil(N / b_kv); the last block may be partial
+ * (its missing key rows are excluded, its missing query rows are not
+ * written).  The bf16 tensor-core kernels work on 128 x 128 tiles; with 64-row
+ * blocks a tile holds two of them and the pairs not listed inside a listed
+ * tile are masked out (their work is computed and discarded). */
 typedef struct {
   int64_t n_tokens;    /* N: rows of the compacted sequence, >= 0 */
   int32_t n_heads;     /* H >= 1 */
   int32_t head_dim;    /* d: 64 or 128 */
-  int32_t block;       /* b: bf16 tensor-core path 128; fp32 path 32, 64, 128 */
+  int32_t block;       /* b_q, rows per query block: bf16 64 or 128; fp32 32, 64, 128 */
   int32_t dtype;       /* ut_dtype of Q, K, V, O, dO, dQ, dK, dV */
   int64_t row_stride;  /* elements between consecutive tokens, >= H*d, multiple of 8 */
+  int32_t block_k;     /* b_kv, rows per key block (Sec. 3.3 sizes the two separately):
+                          0 = same as block; bf16 64 or 128; fp32 equal to block */
 } ut_attn_shape;
 
 const char* ut_strerror(ut_status s);
@@ -263,7 +268,9 @@ ut_status ut_block_mask(const ut_attn_shape* shape, int32_t mode,
 /* ------------------------------------------------------------------------
  * Block-sparse attention forward (Sec. 3.3):
  *   O_i = softmax(Q_i K_{S_i}^T * softmax_scale) V_{S_i}
- * for every head and query block i, S_i the list row_ptr/col_idx gives.
+ * for every head and query block i, S_i the list row_ptr/col_idx gives
+ * (query blocks of b_q rows, listed key blocks of b_kv rows).
+ * A query row whose block lists no key block gets O = 0 and LSE = -inf.
  *   q, k, v, o  [N, H, d] token-major with shape->row_stride (dtype of shape).
  *   lse         [H, N] fp32 natural-log row normalisers (m + log sum exp).
  *   softmax_scale  1/sqrt(d) in the paper; any positive value accepted.

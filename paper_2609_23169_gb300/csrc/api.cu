@@ -69,9 +69,12 @@ static uint64_t wait_timeout_ns() {
 }
 
 // Common checks of an attention shape.  nq_out gets ceil(N / block).
-static ut_status check_shape(const ut_attn_shape* s, int* nq_out) {
+static int block_k_of(const ut_attn_shape* s) { return s->block_k > 0 ? s->block_k : s->block; }
+
+static ut_status check_shape(const ut_attn_shape* s, int* nq_out, int* nk_out = nullptr) {
   if (!s) return UT_ERR_INVALID_ARG;
-  if (s->n_tokens < 0 || s->n_heads < 1 || s->block < 1 || s->head_dim < 1) return UT_ERR_INVALID_ARG;
+  if (s->n_tokens < 0 || s->n_heads < 1 || s->block < 1 || s->head_dim < 1 || s->block_k < 0)
+    return UT_ERR_INVALID_ARG;
   if (s->dtype != UT_BF16 && s->dtype != UT_F32) return UT_ERR_INVALID_ARG;
   if (s->head_dim != 64 && s->head_dim != 128) return UT_ERR_UNSUPPORTED;
   const int64_t hd = (int64_t)s->n_heads * s->head_dim;
@@ -79,14 +82,23 @@ static ut_status check_shape(const ut_attn_shape* s, int* nq_out) {
   if (s->row_stride < hd || (s->row_stride * esz) % 16 != 0) return UT_ERR_INVALID_ARG;
   if (s->n_tokens > INT32_MAX / 2) return UT_ERR_UNSUPPORTED;
   const int64_t nq = (s->n_tokens + s->block - 1) / s->block;
-  if (nq * s->n_heads > INT32_MAX / 2) return UT_ERR_UNSUPPORTED;
+  const int64_t nk = (s->n_tokens + block_k_of(s) - 1) / block_k_of(s);
+  if (nq * s->n_heads > INT32_MAX / 2 || nk * s->n_heads > INT32_MAX / 2) return UT_ERR_UNSUPPORTED;
   *nq_out = (int)nq;
+  if (nk_out) *nk_out = (int)nk;
   return UT_OK;
 }
 
 static bool attn_block_supported(const ut_attn_shape* s) {
-  if (s->dtype == UT_BF16) return s->block == 128;
-  return s->block == 32 || s->block == 64 || s->block == 128;
+  const int bk = block_k_of(s);
+  if (s->dtype == UT_BF16) return (s->block == 64 || s->block == 128) && (bk == 64 || bk == 128);
+  return (s->block == 32 || s->block == 64 || s->block == 128) && bk == s->block;
+}
+
+static AttnProblem attn_problem(const ut_attn_shape* s, int nq, int nk, float scale) {
+  AttnProblem p{s->n_tokens, s->n_heads, s->head_dim, s->block, s->dtype, s->row_stride, nq, scale,
+                block_k_of(s), nk};
+  return p;
 }
 
 }  // namespace ut
@@ -239,8 +251,10 @@ ut_status ut_fg_composite(const uint8_t* mask, int64_t T, void* z, const void* z
 
 size_t ut_block_mask_workspace_size(const ut_attn_shape* shape, int32_t mode) {
   int nq = 0;
-  if (check_shape(shape, &nq) != UT_OK) return 0;
-  MaskProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride, nq};
+  int nk = 0;
+  if (check_shape(shape, &nq, &nk) != UT_OK) return 0;
+  MaskProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride, nq,
+                block_k_of(shape), nk};
   return block_mask_ws(p, mode);
 }
 
@@ -248,14 +262,15 @@ ut_status ut_block_mask(const ut_attn_shape* shape, int32_t mode, const void* q,
                         const uint8_t* bitmap, int32_t* row_ptr, int32_t* col_idx, int64_t col_cap,
                         int32_t* col_ptr_t, int32_t* row_idx_t, void* ws, size_t ws_bytes, int32_t* dev_status,
                         void* stream) {
-  int nq = 0;
-  ut_status st = check_shape(shape, &nq);
+  int nq = 0, nk = 0;
+  ut_status st = check_shape(shape, &nq, &nk);
   if (st != UT_OK) return st;
   if (mode != UT_MASK_TOPK && mode != UT_MASK_BITMAP) return UT_ERR_INVALID_ARG;
   if ((col_ptr_t == nullptr) != (row_idx_t == nullptr)) return UT_ERR_INVALID_ARG;
   if (!row_ptr || col_cap < 0) return UT_ERR_INVALID_ARG;
-  if ((int64_t)nq * nq > (int64_t)1 << 31) return UT_ERR_UNSUPPORTED;
-  MaskProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride, nq};
+  if ((int64_t)nq * nk > (int64_t)1 << 31) return UT_ERR_UNSUPPORTED;
+  MaskProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride, nq,
+                block_k_of(shape), nk};
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (nq == 0) {
     cudaError_t e = cudaMemsetAsync(row_ptr, 0, sizeof(int32_t), s);
@@ -266,7 +281,7 @@ ut_status ut_block_mask(const ut_attn_shape* shape, int32_t mode, const void* q,
   if (mode == UT_MASK_TOPK) {
     if (!(rho > 0.0) || !(rho <= 1.0)) return UT_ERR_INVALID_ARG;
     if (!q || !k || !aligned16(q) || !aligned16(k)) return UT_ERR_INVALID_ARG;
-    const int32_t kr = ut_topk_count(rho, nq);
+    const int32_t kr = ut_topk_count(rho, nk);
     if ((int64_t)shape->n_heads * nq * kr > col_cap || !col_idx) return UT_ERR_CAPACITY;
     return from_cuda(launch_block_mask_topk(p, q, k, kr, row_ptr, col_idx, col_ptr_t, row_idx_t, col_cap, ws,
                                             dev_status, device_sms(), s));
@@ -280,16 +295,15 @@ ut_status ut_block_mask(const ut_attn_shape* shape, int32_t mode, const void* q,
 ut_status ut_bsattn_fwd(const ut_attn_shape* shape, const void* q, const void* k, const void* v,
                         const int32_t* row_ptr, const int32_t* col_idx, float softmax_scale, void* o, float* lse,
                         int32_t* dev_status, void* stream) {
-  int nq = 0;
-  ut_status st = check_shape(shape, &nq);
+  int nq = 0, nk = 0;
+  ut_status st = check_shape(shape, &nq, &nk);
   if (st != UT_OK) return st;
   if (!attn_block_supported(shape)) return UT_ERR_UNSUPPORTED;
   if (!(softmax_scale > 0.f) || !isfinite(softmax_scale)) return UT_ERR_INVALID_ARG;
   if (shape->n_tokens == 0) return UT_OK;
   if (!q || !k || !v || !o || !lse || !row_ptr || !col_idx) return UT_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o)) return UT_ERR_INVALID_ARG;
-  AttnProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride,
-                nq, softmax_scale};
+  const AttnProblem p = attn_problem(shape, nq, nk, softmax_scale);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (shape->dtype == UT_F32) return from_cuda(launch_attn_fwd_simt(p, q, k, v, row_ptr, col_idx, o, lse, s));
   return from_cuda(launch_attn_fwd_tc(p, q, k, v, row_ptr, col_idx, o, lse, dev_status, wait_timeout_ns(),
@@ -297,10 +311,9 @@ ut_status ut_bsattn_fwd(const ut_attn_shape* shape, const void* q, const void* k
 }
 
 size_t ut_bsattn_bwd_workspace_size(const ut_attn_shape* shape) {
-  int nq = 0;
-  if (check_shape(shape, &nq) != UT_OK) return 0;
-  AttnProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride,
-                nq, 1.f};
+  int nq = 0, nk = 0;
+  if (check_shape(shape, &nq, &nk) != UT_OK) return 0;
+  const AttnProblem p = attn_problem(shape, nq, nk, 1.f);
   const size_t a = attn_bwd_simt_ws(p), b = attn_bwd_tc_ws(p);
   return (a > b ? a : b) + 256;
 }
@@ -309,8 +322,8 @@ ut_status ut_bsattn_bwd(const ut_attn_shape* shape, const void* q, const void* k
                         const float* lse, const void* dout, const int32_t* row_ptr, const int32_t* col_idx,
                         const int32_t* col_ptr_t, const int32_t* row_idx_t, float softmax_scale, void* dq, void* dk,
                         void* dv, void* ws, size_t ws_bytes, int32_t* dev_status, void* stream) {
-  int nq = 0;
-  ut_status st = check_shape(shape, &nq);
+  int nq = 0, nk = 0;
+  ut_status st = check_shape(shape, &nq, &nk);
   if (st != UT_OK) return st;
   if (!attn_block_supported(shape)) return UT_ERR_UNSUPPORTED;
   if (!(softmax_scale > 0.f) || !isfinite(softmax_scale)) return UT_ERR_INVALID_ARG;
@@ -318,8 +331,7 @@ ut_status ut_bsattn_bwd(const ut_attn_shape* shape, const void* q, const void* k
   if (!q || !k || !v || !o || !lse || !dout || !row_ptr || !col_idx || !col_ptr_t || !row_idx_t || !dq || !dk ||
       !dv)
     return UT_ERR_INVALID_ARG;
-  AttnProblem p{shape->n_tokens, shape->n_heads, shape->head_dim, shape->block, shape->dtype, shape->row_stride,
-                nq, softmax_scale};
+  const AttnProblem p = attn_problem(shape, nq, nk, softmax_scale);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (shape->dtype == UT_F32) {
     if (!ws || ws_bytes < attn_bwd_simt_ws(p)) return UT_ERR_INVALID_ARG;

@@ -3,23 +3,20 @@
 // With P = exp(S - LSE) recomputed from the forward's row normalisers and
 // D_r = dO_r . O_r:
 //   dV = P^T dO,   dS = P o (dO V^T - D),   dQ = scale * dS K,   dK = scale * dS^T Q
-// over the retained block pairs only.  Two persistent kernels, no atomics:
+// over the retained block pairs only:
 //
-//   bwd_pre_kernel    D_r and LSE_r * log2(e) per (head, row) into a padded
-//                     [H, N_q*128] workspace (padding rows: D = 0, LSE = +inf
-//                     so that they contribute P = 0).
-//   bwd_dq_kernel     item (h, query block i) over its key list S_i:
-//                       S = Q K_j^T, dP = dO V_j^T   (TMEM)
-//                       dS -> bf16, 128B-swizzled shared tile
-//                       dQ += dS K_j                 (TMEM accumulator)
-//   bwd_dkdv_kernel   item (h, key block j) over the transposed list (query
-//                     blocks i with j in S_i):
-//                       S^T = K_j Q_i^T, dP^T = V_j dO_i^T   (TMEM)
-//                       P^T, then dS^T -> bf16 shared tile (one buffer, reused)
-//                       dV += P^T dO_i, dK += dS^T Q_i       (TMEM accumulators)
+//   bwd_pre_kernel          D_r and LSE_r * log2(e) per (head, row) into a
+//                           padded [H, N_t*128] workspace (padding rows: D = 0,
+//                           LSE = +inf so that they contribute P = 0).
+//   bwd_fused_kernel        item (h, 128-row key tile j) over the transposed
+//                           lists: S^T and dP^T once per pair, dK and dV
+//                           accumulated in TMEM, dQ^T partials added into an
+//                           fp32 accumulator (below).
+//   bwd_dq_finalize_kernel  dQ = scale * accumulator, bf16.
 //
-// Roles as in the forward: warp 0 TMA producer, warp 1 TMEM owner + MMA
-// issuer, warps 2-5 elementwise (thread = TMEM lane = one row of the tile).
+// Blocks of 64 rows (b_q or b_kv) are served by the same 128 x 128 tiles: the
+// item's fine lists are merged into 128-row query tiles with a mask of the
+// listed 64 x 64 sub-blocks (TileList); P of unlisted sub-blocks is zero.
 // All waits are bounded (UT_ERR_TIMEOUT on expiry, then drain and return).
 #include "common.cuh"
 #include "kernels.h"
@@ -27,8 +24,6 @@
 namespace ut {
 
 constexpr int kTile = 128;
-constexpr int kDqThreads = 320;    // dQ kernel: 2 role warps + 8 elementwise
-constexpr int kDkdvThreads = 320;  // dK/dV kernel: 2 role warps + 8 elementwise
 constexpr uint32_t kChunk = 128 * 128;  // one 128-row x 128-byte swizzled sub-tile
 
 // ------------------------------------------------------------- preprocess
@@ -69,40 +64,20 @@ __global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __res
 }
 
 struct BwdParams {
-  const int32_t* ptr;   // CSR row_ptr (dq) or CSC col_ptr (dkdv)
-  const int32_t* idx;   // col_idx (dq) or row_idx (dkdv)
+  const int32_t* ptr;   // transposed fine lists: per (head, key block) the query blocks
+  const int32_t* idx;
   const float* lse2;    // [H, Np]  LSE * log2(e)
   const float* dsum;    // [H, Np]  D
-  __nv_bfloat16* out0;  // dq  | dv
-  __nv_bfloat16* out1;  //     | dk
+  __nv_bfloat16* out0;  // dv
+  __nv_bfloat16* out1;  // dk
   int32_t* status;
   int64_t N, Np, rs;
-  int H, nq, n_items;
+  int H, nq, n_items;   // nq: 128-row tiles per head (items = H * nq key tiles)
+  int nk_fine;          // key blocks per head in the transposed lists
+  int k_rows_per_tile;  // 1 (b_kv = 128) or 2 (b_kv = 64)
+  int list_shift;       // 0 (b_q = 128) or 1 (b_q = 64)
   float scale, scale_log2;
   uint64_t timeout_ns;
-};
-
-// =========================================================================
-//                                  dQ
-// =========================================================================
-// dQ kernel rings: K is held from S = Q K^T until dQ += dS K, so it gets the
-// deeper ring; V is released right after dP = dO V^T.  dS lives in TMEM.
-constexpr int kDqKStages = 3, kDqVStages = 2;
-constexpr uint32_t kDqColDs = 384;  // TMEM columns of dS (bf16 pairs): [384, 448)
-
-template <int D>
-struct DqSmem {
-  static constexpr int kC = D / 64;
-  static constexpr uint32_t kTileBytes = kTile * D * 2;
-  alignas(1024) uint8_t q[kTileBytes];
-  alignas(1024) uint8_t dout[kTileBytes];
-  alignas(1024) uint8_t k[kDqKStages][kTileBytes];
-  alignas(1024) uint8_t v[kDqVStages][kTileBytes];
-  uint64_t qd_full, qd_empty;
-  uint64_t k_full[kDqKStages], k_empty[kDqKStages], v_full[kDqVStages], v_empty[kDqVStages];
-  uint64_t s_full, s_empty, dp_full, dp_empty, ds_full, dq_mma_done, dq_empty, mma_done;
-  uint32_t tmem_base;
-  int abort_flag;
 };
 
 // 64 consecutive TMEM columns of this warp's 32 lanes, one wait.
@@ -110,618 +85,6 @@ UT_DEV void tmem_ld64(uint32_t taddr, uint32_t* r) {
   tmem_ld32(taddr, *reinterpret_cast<uint32_t(*)[32]>(r));
   tmem_ld32(taddr + 32, *reinterpret_cast<uint32_t(*)[32]>(r + 32));
   tmem_wait_ld();
-}
-
-template <int D>
-__global__ void __launch_bounds__(kDqThreads, 1)
-    bwd_dq_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                  const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
-                  const BwdParams prm) {
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  DqSmem<D>& sm = *reinterpret_cast<DqSmem<D>*>(smem_raw);
-  constexpr int C = DqSmem<D>::kC;
-  constexpr uint32_t TB = DqSmem<D>::kTileBytes;
-  const uint32_t warp = warp_id(), lane = lane_id();
-  volatile int* abort_flag = &sm.abort_flag;
-  if ((smem_u32(smem_raw) & 1023u) != 0) {  // the swizzled tiles need 1024-byte alignment
-    if (threadIdx.x == 0) set_status(prm.status, UT_ERR_INVALID_ARG);
-    return;
-  }
-  if (threadIdx.x == 0) {
-    mbar_init(&sm.qd_full, 1);
-    mbar_init(&sm.qd_empty, 1);
-    for (int s = 0; s < kDqKStages; ++s) {
-      mbar_init(&sm.k_full[s], 1);
-      mbar_init(&sm.k_empty[s], 1);
-    }
-    for (int s = 0; s < kDqVStages; ++s) {
-      mbar_init(&sm.v_full[s], 1);
-      mbar_init(&sm.v_empty[s], 1);
-    }
-    mbar_init(&sm.s_full, 1);
-    mbar_init(&sm.s_empty, 8);
-    mbar_init(&sm.dp_full, 1);
-    mbar_init(&sm.dp_empty, 8);
-    mbar_init(&sm.ds_full, 8);
-    mbar_init(&sm.dq_mma_done, 1);
-    mbar_init(&sm.dq_empty, 8);
-    mbar_init(&sm.mma_done, 1);
-    sm.abort_flag = 0;
-    fence_barrier_init();
-  }
-  if (warp == 1) {
-    tmem_alloc(&sm.tmem_base, 512);
-    tmem_relinquish();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = sm.tmem_base;
-  const int G = gridDim.x;
-
-  if (warp == 0) {
-    // lane 0: Q, dO and the K ring (K is freed after dQ += dS K);
-    // lane 1: the V ring (V is freed after dP = dO V^T).
-    if (lane < 2) {
-      const bool is_k = lane == 0;
-      if (is_k) {
-        tma_prefetch_desc(&tm_q);
-        tma_prefetch_desc(&tm_k);
-        tma_prefetch_desc(&tm_do);
-      } else {
-        tma_prefetch_desc(&tm_v);
-      }
-      const uint64_t pol_kv = policy_evict_last(), pol_q = policy_evict_first();
-      uint64_t* full = is_k ? sm.k_full : sm.v_full;
-      uint64_t* empty = is_k ? sm.k_empty : sm.v_empty;
-      uint8_t* ring = is_k ? &sm.k[0][0] : &sm.v[0][0];
-      const void* tmap = is_k ? static_cast<const void*>(&tm_k) : static_cast<const void*>(&tm_v);
-      const uint32_t nst = is_k ? kDqKStages : kDqVStages;
-      uint32_t qi = 0, kv = 0;
-      bool ok = true;
-      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-        const int h = w / prm.nq, i = w % prm.nq;
-        const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
-        if (L <= 0) continue;
-        if (is_k) {
-          if (!(ok = mbar_wait(&sm.qd_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          mbar_expect_tx(&sm.qd_full, 2 * TB);
-          for (int c = 0; c < C; ++c) {
-            tma_load_2d(sm.q + c * kChunk, &tm_q, &sm.qd_full, h * D + c * 64, i * kTile, pol_q);
-            tma_load_2d(sm.dout + c * kChunk, &tm_do, &sm.qd_full, h * D + c * 64, i * kTile, pol_q);
-          }
-          ++qi;
-        }
-        for (int t = 0; t < L; ++t, ++kv) {
-          const int j = prm.idx[beg + t];
-          const uint32_t st = kv % nst, n = kv / nst;
-          if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          mbar_expect_tx(&full[st], TB);
-          for (int c = 0; c < C; ++c)
-            tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, j * kTile, pol_kv);
-        }
-      }
-      auto drain = [&](uint64_t* bar, uint32_t parity) {
-        if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
-      };
-      if (qi > 0) drain(&sm.qd_full, (qi - 1) & 1);
-      for (uint32_t u = (kv >= nst ? kv - nst : 0); u < kv; ++u) drain(&full[u % nst], (u / nst) & 1);
-    }
-  } else if (warp == 1) {
-    // whole warp, converged: waits are warp-uniform, MMAs/commits elect one lane
-    {
-      constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
-      constexpr uint32_t idesc_dq = idesc_bf16_f32(kTile, D, false, true);
-      const uint32_t q_addr = smem_u32(sm.q), do_addr = smem_u32(sm.dout);
-      uint32_t qi = 0, kv0 = 0, sc0 = 0;
-      bool ok = true;
-      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-        const int L = prm.ptr[w + 1] - prm.ptr[w];
-        if (L <= 0) continue;
-        if (!(ok = warp_wait(&sm.qd_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        for (int t = 0; t <= L && ok; ++t) {
-          if (t < L) {
-            const uint32_t kv = kv0 + t, sk = kv % kDqKStages, nk = kv / kDqKStages;
-            const uint32_t sv = kv % kDqVStages, nv = kv / kDqVStages;
-            const uint32_t sc = sc0 + t;
-            // S = Q K^T once the previous S has been read; dP = dO V^T once the previous dP has
-            const uint32_t k_addr = smem_u32(sm.k[sk]), v_addr = smem_u32(sm.v[sv]);
-            if (!(ok = warp_wait(&sm.k_full[sk], nk & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = warp_wait(&sm.s_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            tc_fence_after();
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024), idesc_s,
-                          kk > 0);
-            }
-            mma_commit_w(&sm.s_full);
-            if (!(ok = warp_wait(&sm.v_full[sv], nv & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (!(ok = warp_wait(&sm.dp_empty, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            tc_fence_after();
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-              mma_bf16_ss_w(tmem + 128, sdesc_sw128(do_addr + off, 16, 1024), sdesc_sw128(v_addr + off, 16, 1024),
-                          idesc_s, kk > 0);
-            }
-            mma_commit_w(&sm.dp_full);
-            mma_commit_w(&sm.v_empty[sv]);
-            if (t == L - 1) mma_commit_w(&sm.qd_empty);
-          }
-          if (t >= 1) {
-            const uint32_t u = t - 1;
-            const uint32_t kv = kv0 + u, sk = kv % kDqKStages;
-            const uint32_t sc = sc0 + u;
-            if (!(ok = warp_wait(&sm.ds_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-            if (u == 0 && !(ok = warp_wait(&sm.dq_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
-              break;
-            tc_fence_after();
-            const uint32_t k_addr = smem_u32(sm.k[sk]);
-#pragma unroll
-            for (int kk = 0; kk < kTile / 16; ++kk)
-              mma_bf16_ts_w(tmem + 256, tmem + kDqColDs + kk * 8, sdesc_sw128(k_addr + kk * 2048, kChunk, 1024),
-                            idesc_dq, (u > 0 || kk > 0));
-            mma_commit_w(&sm.dq_mma_done);
-            mma_commit_w(&sm.k_empty[sk]);
-          }
-        }
-        kv0 += L;
-        sc0 += L;
-        ++qi;
-      }
-      mma_commit_w(&sm.mma_done);
-      if (!mbar_drain(&sm.mma_done, 0, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
-    }
-  } else {
-    // 8 elementwise warps: warps w and w+4 share TMEM lane quarter (w & 3),
-    // i.e. the same 32 query rows, and split the 128 key columns (and the D
-    // output columns) into halves; a half is one 128-byte swizzle chunk of dS.
-    const uint32_t quarter = warp & 3;
-    const uint32_t half = (warp - 2) >> 2;
-    const uint32_t row = quarter * 32 + lane;
-    const uint32_t lane_base = (quarter * 32) << 16;
-    constexpr int HC = kTile / 2;
-    constexpr int HD = D / 2;
-    const float c = prm.scale_log2;
-    uint32_t sc0 = 0;
-    bool ok = true;
-    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-      const int h = w / prm.nq, i = w % prm.nq;
-      const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
-      const int64_t grow = (int64_t)i * kTile + row;
-      const bool row_ok = grow < prm.N;
-      __nv_bfloat16* orow = prm.out0 + grow * prm.rs + (int64_t)h * D + half * HD;
-      if (L <= 0) {
-        if (row_ok)
-          for (int e = 0; e < HD; e += 8) *reinterpret_cast<uint4*>(orow + e) = make_uint4(0, 0, 0, 0);
-        continue;
-      }
-      const float lse2 = prm.lse2[(int64_t)h * prm.Np + grow];
-      const float Dr = prm.dsum[(int64_t)h * prm.Np + grow];
-      int j_cur = prm.idx[beg];
-      for (int t = 0; t < L; ++t) {
-        const uint32_t sc = sc0 + t;
-        const int j = j_cur;
-        if (t + 1 < L) j_cur = prm.idx[beg + t + 1];  // prefetch the next key block index
-        const int64_t nv = prm.N - (int64_t)j * kTile - (int64_t)half * HC;  // valid columns of this half
-        if (!(ok = warp_wait(&sm.s_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        tc_fence_after();
-        float p[HC];
-        {
-          uint32_t r[HC];
-          tmem_ld64(tmem + lane_base + half * HC, r);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&sm.s_empty);
-#pragma unroll
-          for (int x = 0; x < HC; ++x) p[x] = ex2_approx(fmaf(__uint_as_float(r[x]), c, -lse2));
-          if (nv < HC) {  // ragged last key block: columns past N do not exist
-#pragma unroll
-            for (int x = 0; x < HC; ++x)
-              if (x >= nv) p[x] = 0.f;
-          }
-        }
-        if (!(ok = warp_wait(&sm.dp_full, sc & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        tc_fence_after();
-        // dS buffer is free once the previous tile's dQ MMA finished
-        if (!(ok = warp_wait(&sm.dq_mma_done, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        tc_fence_after();
-        {
-          uint32_t r[HC];
-          tmem_ld64(tmem + lane_base + 128 + half * HC, r);
-          uint32_t pk[HC / 2];
-#pragma unroll
-          for (int x = 0; x < HC; x += 2)
-            pk[x / 2] = pack_bf16x2(p[x] * (__uint_as_float(r[x]) - Dr), p[x + 1] * (__uint_as_float(r[x + 1]) - Dr));
-          // dS (bf16 pairs) into TMEM: this half's 64 keys are columns [kDqColDs + 32*half, +32)
-          tmem_st32(tmem + lane_base + kDqColDs + half * (HC / 2), pk);
-          tmem_wait_st();
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&sm.dp_empty);
-          mbar_arrive(&sm.ds_full);
-        }
-      }
-      if (!ok) break;
-      const uint32_t last = sc0 + L - 1;
-      if (!(ok = warp_wait(&sm.dq_mma_done, last & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-      tc_fence_after();
-#pragma unroll
-      for (int g = 0; g < HD / 32; ++g) {
-        uint32_t r[32];
-        tmem_ld32(tmem + lane_base + 256 + half * HD + g * 32, r);
-        tmem_wait_ld();
-        if (row_ok) {
-#pragma unroll
-          for (int x = 0; x < 32; x += 8) {
-            uint4 v;
-            v.x = pack_bf16x2(__uint_as_float(r[x + 0]) * prm.scale, __uint_as_float(r[x + 1]) * prm.scale);
-            v.y = pack_bf16x2(__uint_as_float(r[x + 2]) * prm.scale, __uint_as_float(r[x + 3]) * prm.scale);
-            v.z = pack_bf16x2(__uint_as_float(r[x + 4]) * prm.scale, __uint_as_float(r[x + 5]) * prm.scale);
-            v.w = pack_bf16x2(__uint_as_float(r[x + 6]) * prm.scale, __uint_as_float(r[x + 7]) * prm.scale);
-            *reinterpret_cast<uint4*>(orow + g * 32 + x) = v;
-          }
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.dq_empty);
-      sc0 += L;
-    }
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, 512);
-}
-
-// =========================================================================
-//                                dK, dV
-// =========================================================================
-// TMEM columns (512): S^T and then dP^T of a pair share [0,128) (dP^T is
-// computed once S^T has been read), P^T bf16 pairs [128,192), dS^T bf16 pairs
-// [192,256), dV accumulator [256,384), dK accumulator [384,512).  dV += P^T dO
-// and dK += dS^T Q read their A operand from TMEM (TS form).
-constexpr int kKvQStages = 3, kKvDoStages = 2;
-constexpr uint32_t kColSdp = 0, kColPt = 128, kColDst = 192, kColDv = 256, kColDk = 384;
-
-template <int D>
-struct DkdvSmem {
-  static constexpr int kC = D / 64;
-  static constexpr uint32_t kTileBytes = kTile * D * 2;
-  alignas(1024) uint8_t k[kTileBytes];
-  alignas(1024) uint8_t v[kTileBytes];
-  alignas(1024) uint8_t q[kKvQStages][kTileBytes];
-  alignas(1024) uint8_t dout[kKvDoStages][kTileBytes];
-  alignas(16) float lse2[2][kTile];
-  alignas(16) float dsum[2][kTile];
-  uint64_t kv_full, kv_empty;
-  uint64_t q_full[kKvQStages], q_empty[kKvQStages], do_full[kKvDoStages], do_empty[kKvDoStages];
-  uint64_t s_full, s_empty, dp_full, dp_empty, pt_full, pt_done, dst_full, ds_done, acc_full, acc_empty, mma_done;
-  uint64_t rowvec_full[2];   // the elementwise threads staged this pair's LSE / D
-  uint32_t tmem_base;
-  int abort_flag;
-};
-
-template <int D>
-__global__ void __launch_bounds__(kDkdvThreads, 1)
-    bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
-                    const BwdParams prm) {
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  DkdvSmem<D>& sm = *reinterpret_cast<DkdvSmem<D>*>(smem_raw);
-  constexpr int C = DkdvSmem<D>::kC;
-  constexpr uint32_t TB = DkdvSmem<D>::kTileBytes;
-  const uint32_t warp = warp_id(), lane = lane_id();
-  volatile int* abort_flag = &sm.abort_flag;
-  if ((smem_u32(smem_raw) & 1023u) != 0) {
-    if (threadIdx.x == 0) set_status(prm.status, UT_ERR_INVALID_ARG);
-    return;
-  }
-  if (threadIdx.x == 0) {
-    mbar_init(&sm.kv_full, 1);
-    mbar_init(&sm.kv_empty, 1);
-    for (int s = 0; s < kKvQStages; ++s) {
-      mbar_init(&sm.q_full[s], 1);
-      mbar_init(&sm.q_empty[s], 1);
-    }
-    for (int s = 0; s < kKvDoStages; ++s) {
-      mbar_init(&sm.do_full[s], 1);
-      mbar_init(&sm.do_empty[s], 1);
-    }
-    mbar_init(&sm.s_full, 1);
-    mbar_init(&sm.s_empty, 8);
-    mbar_init(&sm.dp_full, 1);
-    mbar_init(&sm.dp_empty, 8);
-    mbar_init(&sm.pt_full, 8);
-    mbar_init(&sm.pt_done, 1);
-    mbar_init(&sm.dst_full, 8);
-    mbar_init(&sm.ds_done, 1);
-    mbar_init(&sm.acc_full, 1);
-    mbar_init(&sm.acc_empty, 8);
-    mbar_init(&sm.mma_done, 1);
-    mbar_init(&sm.rowvec_full[0], 256);
-    mbar_init(&sm.rowvec_full[1], 256);
-    sm.abort_flag = 0;
-    fence_barrier_init();
-  }
-  if (warp == 1) {
-    tmem_alloc(&sm.tmem_base, 512);
-    tmem_relinquish();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = sm.tmem_base;
-  const int G = gridDim.x;
-
-  if (warp == 0) {
-    // lane 0: K, V of the item and the Q ring (Q is freed after dK += dS^T Q);
-    // lane 1: the dO ring (dO is freed after dV += P^T dO).
-    if (lane < 2) {
-      const bool is_q = lane == 0;
-      if (is_q) {
-        tma_prefetch_desc(&tm_q);
-        tma_prefetch_desc(&tm_k);
-        tma_prefetch_desc(&tm_v);
-      } else {
-        tma_prefetch_desc(&tm_do);
-      }
-      const uint64_t pol_qd = policy_evict_last(), pol_kv = policy_evict_first();
-      uint64_t* full = is_q ? sm.q_full : sm.do_full;
-      uint64_t* empty = is_q ? sm.q_empty : sm.do_empty;
-      uint8_t* ring = is_q ? &sm.q[0][0] : &sm.dout[0][0];
-      const void* tmap = is_q ? static_cast<const void*>(&tm_q) : static_cast<const void*>(&tm_do);
-      const uint32_t nst = is_q ? kKvQStages : kKvDoStages;
-      uint32_t ki = 0, qd = 0;
-      bool ok = true;
-      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-        const int h = w / prm.nq, j = w % prm.nq;
-        const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
-        if (L <= 0) continue;
-        if (is_q) {
-          if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          mbar_expect_tx(&sm.kv_full, 2 * TB);
-          for (int c = 0; c < C; ++c) {
-            tma_load_2d(sm.k + c * kChunk, &tm_k, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
-            tma_load_2d(sm.v + c * kChunk, &tm_v, &sm.kv_full, h * D + c * 64, j * kTile, pol_kv);
-          }
-          ++ki;
-        }
-        for (int t = 0; t < L; ++t, ++qd) {
-          const int i = prm.idx[beg + t];
-          const uint32_t st = qd % nst, n = qd / nst;
-          if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          mbar_expect_tx(&full[st], TB);
-          for (int c = 0; c < C; ++c)
-            tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, i * kTile, pol_qd);
-        }
-      }
-      auto drain = [&](uint64_t* bar, uint32_t parity) {
-        if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
-      };
-      if (ki > 0) drain(&sm.kv_full, (ki - 1) & 1);
-      for (uint32_t u = (qd >= nst ? qd - nst : 0); u < qd; ++u) drain(&full[u % nst], (u / nst) & 1);
-    }
-  } else if (warp == 1) {
-    // whole warp, converged: waits are warp-uniform, MMAs/commits elect one lane.
-    // Per pair t: dP^T_t (after S^T_t was read), dV_t (after P^T_t is in TMEM),
-    // S^T_{t+1} (after dP^T_t was read), dK_t (after dS^T_t is in TMEM).
-    {
-      constexpr uint32_t idesc_s = idesc_bf16_f32(kTile, kTile, false, false);
-      constexpr uint32_t idesc_acc = idesc_bf16_f32(kTile, D, false, true);
-      const uint32_t k_addr = smem_u32(sm.k), v_addr = smem_u32(sm.v);
-      uint32_t ki = 0, qd0 = 0;
-      bool ok = true;
-      for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-        const int L = prm.ptr[w + 1] - prm.ptr[w];
-        if (L <= 0) continue;
-        if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        auto issue_st = [&](int t) -> bool {  // S^T_t = K Q_t^T into [0,128)
-          const uint32_t qd = qd0 + t, st = qd % kKvQStages, n = qd / kKvQStages;
-          if (!warp_wait(&sm.q_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
-          if (!warp_wait(&sm.dp_empty, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)) return false;
-          tc_fence_after();
-          const uint32_t q_addr = smem_u32(sm.q[st]);
-#pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-            mma_bf16_ss_w(tmem + kColSdp, sdesc_sw128(k_addr + off, 16, 1024), sdesc_sw128(q_addr + off, 16, 1024),
-                          idesc_s, kk > 0);
-          }
-          mma_commit_w(&sm.s_full);
-          return true;
-        };
-        if (!(ok = issue_st(0))) break;
-        for (int t = 0; t < L && ok; ++t) {
-          const uint32_t qd = qd0 + t;
-          const uint32_t sq = qd % kKvQStages, sd = qd % kKvDoStages, nd = qd / kKvDoStages;
-          // dP^T_t = V dO_t^T into [0,128) once S^T_t has been read
-          if (!(ok = warp_wait(&sm.do_full[sd], nd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          if (!(ok = warp_wait(&sm.s_empty, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          tc_fence_after();
-          const uint32_t do_addr = smem_u32(sm.dout[sd]);
-#pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * kChunk + (kk & 3) * 32;
-            mma_bf16_ss_w(tmem + kColSdp, sdesc_sw128(v_addr + off, 16, 1024), sdesc_sw128(do_addr + off, 16, 1024),
-                          idesc_s, kk > 0);
-          }
-          mma_commit_w(&sm.dp_full);
-          if (t == L - 1) mma_commit_w(&sm.kv_empty);
-          // dV += P^T_t dO_t
-          if (!(ok = warp_wait(&sm.pt_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          if (t == 0 && !(ok = warp_wait(&sm.acc_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)))
-            break;
-          tc_fence_after();
-#pragma unroll
-          for (int kk = 0; kk < kTile / 16; ++kk)
-            mma_bf16_ts_w(tmem + kColDv, tmem + kColPt + kk * 8, sdesc_sw128(do_addr + kk * 2048, kChunk, 1024),
-                          idesc_acc, (t > 0 || kk > 0));
-          mma_commit_w(&sm.pt_done);
-          mma_commit_w(&sm.do_empty[sd]);
-          // S^T_{t+1} once dP^T_t has been read
-          if (t + 1 < L && !(ok = issue_st(t + 1))) break;
-          // dK += dS^T_t Q_t
-          if (!(ok = warp_wait(&sm.dst_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          tc_fence_after();
-          const uint32_t q_addr = smem_u32(sm.q[sq]);
-#pragma unroll
-          for (int kk = 0; kk < kTile / 16; ++kk)
-            mma_bf16_ts_w(tmem + kColDk, tmem + kColDst + kk * 8, sdesc_sw128(q_addr + kk * 2048, kChunk, 1024),
-                          idesc_acc, (t > 0 || kk > 0));
-          mma_commit_w(&sm.ds_done);
-          mma_commit_w(&sm.q_empty[sq]);
-        }
-        mma_commit_w(&sm.acc_full);
-        qd0 += L;
-        ++ki;
-      }
-      mma_commit_w(&sm.mma_done);
-      if (!mbar_drain(&sm.mma_done, 0, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
-    }
-  } else {
-    // 8 elementwise warps: warps w and w+4 share TMEM lane quarter (w & 3),
-    // i.e. the same 32 key rows, and split the 128 query columns (and the D
-    // output columns) into halves.
-    const uint32_t quarter = warp & 3;
-    const uint32_t half = (warp - 2) >> 2;
-    const uint32_t krow = quarter * 32 + lane;          // key row of the tile = TMEM lane
-    const uint32_t tid = threadIdx.x - 64;               // 0..255 within the elementwise group
-    const uint32_t lane_base = (quarter * 32) << 16;
-    constexpr int HC = kTile / 2;                        // query columns per half
-    constexpr int HD = D / 2;                            // output columns per half
-    const float c = prm.scale_log2;
-    uint32_t qd0 = 0, ki = 0;
-    bool ok = true;
-    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-      const int h = w / prm.nq, j = w % prm.nq;
-      const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
-      const int64_t gk = (int64_t)j * kTile + krow;
-      const bool row_ok = gk < prm.N;
-      __nv_bfloat16* dv_row = prm.out0 + gk * prm.rs + (int64_t)h * D + half * HD;
-      __nv_bfloat16* dk_row = prm.out1 + gk * prm.rs + (int64_t)h * D + half * HD;
-      if (L <= 0) {
-        if (row_ok)
-          for (int e = 0; e < HD; e += 8) {
-            *reinterpret_cast<uint4*>(dv_row + e) = make_uint4(0, 0, 0, 0);
-            *reinterpret_cast<uint4*>(dk_row + e) = make_uint4(0, 0, 0, 0);
-          }
-        continue;
-      }
-      // this thread's element of the query-row vectors (LSE*log2e for threads
-      // 0-127, D for 128-255) is loaded one pair ahead
-      const float* rv_src = (tid < kTile ? prm.lse2 + tid : prm.dsum + (tid - kTile)) + (int64_t)h * prm.Np;
-      float rv = rv_src[(int64_t)prm.idx[beg] * kTile];
-      for (int t = 0; t < L; ++t) {
-        const uint32_t qd = qd0 + t;
-        // this pair's query-row LSE*log2e and D into the shared double buffer
-        // (buffer qd&1 was last read in pair qd-2, which every thread finished
-        //  before arriving for pair qd-1)
-        if (tid < kTile) sm.lse2[qd & 1][tid] = rv;
-        else sm.dsum[qd & 1][tid - kTile] = rv;
-        mbar_arrive(&sm.rowvec_full[qd & 1]);
-        if (t + 1 < L) rv = rv_src[(int64_t)prm.idx[beg + t + 1] * kTile];
-        if (!(ok = warp_wait(&sm.rowvec_full[qd & 1], (qd >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
-          break;
-        const float* ls = sm.lse2[qd & 1] + half * HC;
-        const float* ds_v = sm.dsum[qd & 1] + half * HC;
-        if (!(ok = warp_wait(&sm.s_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        tc_fence_after();
-        float p[HC];
-        {
-          uint32_t r[HC];
-          tmem_ld64(tmem + lane_base + kColSdp + half * HC, r);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&sm.s_empty);
-#pragma unroll
-          for (int x = 0; x < HC; x += 4) {
-            const float4 l4 = *reinterpret_cast<const float4*>(ls + x);
-            p[x + 0] = ex2_approx(fmaf(__uint_as_float(r[x + 0]), c, -l4.x));
-            p[x + 1] = ex2_approx(fmaf(__uint_as_float(r[x + 1]), c, -l4.y));
-            p[x + 2] = ex2_approx(fmaf(__uint_as_float(r[x + 2]), c, -l4.z));
-            p[x + 3] = ex2_approx(fmaf(__uint_as_float(r[x + 3]), c, -l4.w));
-          }
-        }
-        {
-          uint32_t pk[HC / 2];
-#pragma unroll
-          for (int x = 0; x < HC; x += 2) pk[x / 2] = pack_bf16x2(p[x], p[x + 1]);
-          // the TMEM P^T region is free once the previous pair's dV MMA finished
-          if (!(ok = warp_wait(&sm.pt_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          tc_fence_after();
-          tmem_st32(tmem + lane_base + kColPt + half * (HC / 2), pk);
-          tmem_wait_st();
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.pt_full);
-        if (!(ok = warp_wait(&sm.dp_full, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-        tc_fence_after();
-        {
-          uint32_t r[HC];
-          tmem_ld64(tmem + lane_base + kColSdp + half * HC, r);
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&sm.dp_empty);
-          uint32_t dsk[HC / 2];
-#pragma unroll
-          for (int x = 0; x < HC; x += 4) {
-            const float4 d4 = *reinterpret_cast<const float4*>(ds_v + x);
-            dsk[x / 2] = pack_bf16x2(p[x] * (__uint_as_float(r[x]) - d4.x), p[x + 1] * (__uint_as_float(r[x + 1]) - d4.y));
-            dsk[x / 2 + 1] =
-                pack_bf16x2(p[x + 2] * (__uint_as_float(r[x + 2]) - d4.z), p[x + 3] * (__uint_as_float(r[x + 3]) - d4.w));
-          }
-          // the TMEM dS^T region is free once the previous pair's dK MMA finished
-          if (!(ok = warp_wait(&sm.ds_done, (qd & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
-          tc_fence_after();
-          tmem_st32(tmem + lane_base + kColDst + half * (HC / 2), dsk);
-          tmem_wait_st();
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.dst_full);
-      }
-      if (!ok) break;
-      if (!(ok = warp_wait(&sm.acc_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-      tc_fence_after();
-#pragma unroll
-      for (int part = 0; part < 2; ++part) {
-        __nv_bfloat16* dst = part == 0 ? dv_row : dk_row;
-        const float f = part == 0 ? 1.0f : prm.scale;
-#pragma unroll
-        for (int g = 0; g < HD / 32; ++g) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_base + (part == 0 ? kColDv : kColDk) + half * HD + g * 32, r);
-          tmem_wait_ld();
-          if (row_ok) {
-#pragma unroll
-            for (int x = 0; x < 32; x += 8) {
-              uint4 v;
-              v.x = pack_bf16x2(__uint_as_float(r[x + 0]) * f, __uint_as_float(r[x + 1]) * f);
-              v.y = pack_bf16x2(__uint_as_float(r[x + 2]) * f, __uint_as_float(r[x + 3]) * f);
-              v.z = pack_bf16x2(__uint_as_float(r[x + 4]) * f, __uint_as_float(r[x + 5]) * f);
-              v.w = pack_bf16x2(__uint_as_float(r[x + 6]) * f, __uint_as_float(r[x + 7]) * f);
-              *reinterpret_cast<uint4*>(dst + g * 32 + x) = v;
-            }
-          }
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.acc_empty);
-      qd0 += L;
-      ++ki;
-    }
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
 // =========================================================================
@@ -783,7 +146,7 @@ UT_DEV void red_add_f32(float* p, float v) {
   asm volatile("red.relaxed.gpu.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
 }
 
-template <int D>
+template <int D, bool kSub>
 __global__ void __launch_bounds__(kFuThreads, 1)
     bwd_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
@@ -865,7 +228,9 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         bool ok = true;
         for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
           const int h = w / prm.nq, j = w % prm.nq;
-          const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+          TileList<kSub> tl;
+          tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+          const int L = tl.count();
           if (L <= 0) continue;
           if (is_q) {
             if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -877,7 +242,9 @@ __global__ void __launch_bounds__(kFuThreads, 1)
             ++ki;
           }
           for (int t = 0; t < L; ++t, ++qd) {
-            const int i = prm.idx[beg + t];
+            int i;
+            uint32_t bits;
+            tl.next(i, bits);
             const uint32_t st = qd % nst, n = qd / nst;
             if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             mbar_expect_tx(&full[st], TB);
@@ -903,7 +270,9 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         uint32_t ki = 0, qd0 = 0;
         bool ok = true;
         for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-          const int L = prm.ptr[w + 1] - prm.ptr[w];
+          TileList<kSub> tl;
+          tl.init(prm.ptr, prm.idx, w / prm.nq, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+          const int L = tl.count();
           if (L <= 0) continue;
           if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
           auto issue_st = [&](int t) -> bool {  // S^T_t = K Q_t^T into R0
@@ -997,9 +366,12 @@ __global__ void __launch_bounds__(kFuThreads, 1)
     const uint32_t dst_row = smem_u32(sm.dst) + half * kChunk + krow * 128;
     uint32_t qd0 = 0, ki = 0;
     bool ok = true;
+    const uint32_t kh = krow >> 6;  // which 64-row half of the key tile
     for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
       const int h = w / prm.nq, j = w % prm.nq;
-      const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+      TileList<kSub> tl;
+      tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+      const int L = tl.count();
       const int64_t gk = (int64_t)j * kTile + krow;
       const bool row_ok = gk < prm.N;
       __nv_bfloat16* dv_row = prm.out0 + gk * prm.rs + (int64_t)h * D + half * HD;
@@ -1015,16 +387,22 @@ __global__ void __launch_bounds__(kFuThreads, 1)
       // this thread's element of the query-row vectors (LSE*log2e for threads
       // 0-127, D for 128-255) is loaded one pair ahead
       const float* rv_src = (tid < kTile ? prm.lse2 + tid : prm.dsum + (tid - kTile)) + (int64_t)h * prm.Np;
-      float rv = rv_src[(int64_t)prm.idx[beg] * kTile];
+      int i_next;
+      uint32_t bits_next;
+      tl.next(i_next, bits_next);
+      float rv = rv_src[(int64_t)i_next * kTile];
       for (int t = 0; t < L; ++t) {
         const uint32_t qd = qd0 + t;
+        // this half's 64 query columns and this thread's 64 key rows form one
+        // 64 x 64 sub-block of the tile pair: listed or not
+        const bool listed = !kSub || ((bits_next >> (2 * kh + half)) & 1u);
         // this pair's query-row LSE*log2e and D into the shared double buffer
         // (buffer qd&1 was last read in pair qd-2, which every thread finished
         //  before arriving for pair qd-1)
         if (tid < kTile) sm.lse2[qd & 1][tid] = rv;
         else sm.dsum[qd & 1][tid - kTile] = rv;
         mbar_arrive(&sm.rowvec_full[qd & 1]);
-        if (t + 1 < L) rv = rv_src[(int64_t)prm.idx[beg + t + 1] * kTile];
+        if (t + 1 < L && tl.next(i_next, bits_next)) rv = rv_src[(int64_t)i_next * kTile];
         if (!(ok = warp_wait(&sm.rowvec_full[qd & 1], (qd >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
           break;
         const float* ls = sm.lse2[qd & 1] + half * HC;
@@ -1038,13 +416,18 @@ __global__ void __launch_bounds__(kFuThreads, 1)
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&sm.s_empty);
+          if (listed) {
 #pragma unroll
-          for (int x = 0; x < HC; x += 4) {
-            const float4 l4 = *reinterpret_cast<const float4*>(ls + x);
-            p[x + 0] = ex2_approx(fmaf(__uint_as_float(r[x + 0]), c, -l4.x));
-            p[x + 1] = ex2_approx(fmaf(__uint_as_float(r[x + 1]), c, -l4.y));
-            p[x + 2] = ex2_approx(fmaf(__uint_as_float(r[x + 2]), c, -l4.z));
-            p[x + 3] = ex2_approx(fmaf(__uint_as_float(r[x + 3]), c, -l4.w));
+            for (int x = 0; x < HC; x += 4) {
+              const float4 l4 = *reinterpret_cast<const float4*>(ls + x);
+              p[x + 0] = ex2_approx(fmaf(__uint_as_float(r[x + 0]), c, -l4.x));
+              p[x + 1] = ex2_approx(fmaf(__uint_as_float(r[x + 1]), c, -l4.y));
+              p[x + 2] = ex2_approx(fmaf(__uint_as_float(r[x + 2]), c, -l4.z));
+              p[x + 3] = ex2_approx(fmaf(__uint_as_float(r[x + 3]), c, -l4.w));
+            }
+          } else {
+#pragma unroll
+            for (int x = 0; x < HC; ++x) p[x] = 0.f;
           }
         }
         // the P^T tile is free once the previous pair's dV MMA finished
@@ -1138,11 +521,15 @@ __global__ void __launch_bounds__(kFuThreads, 1)
     bool ok = true;
     for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
       const int h = w / prm.nq;
-      const int beg = prm.ptr[w], L = prm.ptr[w + 1] - beg;
+      TileList<kSub> tl;
+      tl.init(prm.ptr, prm.idx, h, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+      const int L = tl.count();
       if (L <= 0) continue;
       for (int t = 0; t < L; ++t) {
         const uint32_t qd = qd0 + t;
-        const int i = prm.idx[beg + t];
+        int i;
+        uint32_t bits;
+        tl.next(i, bits);
         if (!(ok = warp_wait(&sm.ds_done, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
         float* dst = dq_acc + (((int64_t)h * prm.Np + (int64_t)i * kTile) * D + dcol);
@@ -1191,60 +578,35 @@ __global__ void __launch_bounds__(256) bwd_dq_finalize_kernel(const float* __res
 }
 
 // ----------------------------------------------------------------- launcher
-// The fused kernel replaces the dQ and dK/dV kernel pair (it computes S and dP
-// once per block pair instead of twice) at the cost of an fp32 dQ accumulator
-// in the workspace.
-constexpr bool kFusedBwd = true;
-
 size_t attn_bwd_tc_ws(const AttnProblem& p) {
-  const size_t Np = (size_t)p.nq * kTile;
-  return 2 * (size_t)p.H * Np * sizeof(float) + (kFusedBwd ? (size_t)p.H * Np * p.d * sizeof(float) : 0);
+  const size_t Np = (size_t)((p.N + kTile - 1) / kTile) * kTile;
+  return 2 * (size_t)p.H * Np * sizeof(float) + (size_t)p.H * Np * p.d * sizeof(float);
 }
 
 constexpr size_t kMaxDynSmem = 232448;  // 227 KB opt-in per block on sm_100/sm_103
-static_assert(sizeof(DqSmem<128>) <= kMaxDynSmem, "dQ shared layout exceeds the per-block limit");
-static_assert(kDqColDs + kTile / 2 <= 512, "dQ TMEM columns");
-static_assert(sizeof(DkdvSmem<128>) <= kMaxDynSmem, "dK/dV shared layout exceeds the per-block limit");
 static_assert(sizeof(FusedSmem<128>) <= kMaxDynSmem, "fused backward shared layout exceeds the per-block limit");
 
-template <int D>
+template <int D, bool kSub>
 static cudaError_t launch_bwd_fused(const AttnProblem& p, const CUtensorMap* tm, BwdParams prm, float* dq_acc,
                                    __nv_bfloat16* dq, int sms, cudaStream_t s) {
-  const int n_items = p.H * p.nq;
+  const int n_items = prm.n_items;
   const int grid = n_items < sms ? n_items : sms;
   const size_t smem = sizeof(FusedSmem<D>);
-  cudaError_t e = cudaFuncSetAttribute(bwd_fused_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e =
+      cudaFuncSetAttribute(bwd_fused_kernel<D, kSub>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   // the setmaxnreg split assumes exactly kFuRegLaunch registers per thread at
   // launch: with fewer, the increases would wait for registers that never come
   cudaFuncAttributes fa;
-  e = cudaFuncGetAttributes(&fa, bwd_fused_kernel<D>);
+  e = cudaFuncGetAttributes(&fa, bwd_fused_kernel<D, kSub>);
   if (e != cudaSuccess) return e;
   if (fa.numRegs != kFuRegLaunch) return cudaErrorInvalidConfiguration;
-  bwd_fused_kernel<D><<<grid, kFuThreads, smem, s>>>(tm[0], tm[1], tm[2], tm[3], prm, dq_acc);
+  bwd_fused_kernel<D, kSub><<<grid, kFuThreads, smem, s>>>(tm[0], tm[1], tm[2], tm[3], prm, dq_acc);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int64_t n8 = p.N * p.H * D / 8;
-  bwd_dq_finalize_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, s>>>(dq_acc, p.N, (int64_t)p.nq * kTile, p.H, D,
-                                                                      p.row_stride, p.scale, dq);
-  return cudaGetLastError();
-}
-
-template <int D>
-static cudaError_t launch_bwd_d(const AttnProblem& p, const CUtensorMap* tm, BwdParams prm_dq, BwdParams prm_kv,
-                                int sms, cudaStream_t s) {
-  const int n_items = p.H * p.nq;
-  const int grid = n_items < sms ? n_items : sms;
-  const size_t smem_dq = sizeof(DqSmem<D>);
-  const size_t smem_kv = sizeof(DkdvSmem<D>);
-  cudaError_t e = cudaFuncSetAttribute(bwd_dq_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_dq);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(bwd_dkdv_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_kv);
-  if (e != cudaSuccess) return e;
-  bwd_dkdv_kernel<D><<<grid, kDkdvThreads, smem_kv, s>>>(tm[0], tm[1], tm[2], tm[3], prm_kv);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  bwd_dq_kernel<D><<<grid, kDqThreads, smem_dq, s>>>(tm[0], tm[1], tm[2], tm[3], prm_dq);
+  bwd_dq_finalize_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, s>>>(dq_acc, p.N, prm.Np, p.H, D, p.row_stride,
+                                                                      p.scale, dq);
   return cudaGetLastError();
 }
 
@@ -1252,19 +614,20 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
                                const float* lse, const void* dout, const int32_t* row_ptr, const int32_t* col_idx,
                                const int32_t* col_ptr_t, const int32_t* row_idx_t, void* dq, void* dk, void* dv,
                                void* ws, int32_t* status, uint64_t timeout_ns, int sms, cudaStream_t stream) {
-  if (p.nq == 0) return cudaSuccess;
-  const int64_t Np = (int64_t)p.nq * kTile;
+  (void)row_ptr;
+  (void)col_idx;  // the fused kernel walks the transposed lists only
+  const int nt = (int)((p.N + kTile - 1) / kTile);  // 128-row tiles
+  if (nt == 0) return cudaSuccess;
+  const int64_t Np = (int64_t)nt * kTile;
   float* lse2 = static_cast<float*>(ws);
   float* dsum = lse2 + (size_t)p.H * Np;
   float* dq_acc = dsum + (size_t)p.H * Np;
-  if (kFusedBwd) {
-    cudaError_t e0 = cudaMemsetAsync(dq_acc, 0, (size_t)p.H * Np * p.d * sizeof(float), stream);
-    if (e0 != cudaSuccess) return e0;
-  }
+  cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)p.H * Np * p.d * sizeof(float), stream);
+  if (e != cudaSuccess) return e;
   bwd_pre_kernel<<<(unsigned)((Np + 7) / 8), 256, 0, stream>>>(
       static_cast<const __nv_bfloat16*>(o), static_cast<const __nv_bfloat16*>(dout), lse, p.N, Np, p.H, p.d,
       p.row_stride, lse2, dsum);
-  cudaError_t e = cudaGetLastError();
+  e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   CUtensorMap tm[4];
   const uint64_t inner = (uint64_t)p.H * p.d, stride = (uint64_t)p.row_stride * 2;
@@ -1272,30 +635,32 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
   for (int x = 0; x < 4; ++x)
     if (!encode_tmap_2d_bf16(&tm[x], bases[x], inner, p.N, stride, 64, kTile)) return cudaErrorInvalidValue;
   BwdParams a{};
+  a.ptr = col_ptr_t;
+  a.idx = row_idx_t;
   a.lse2 = lse2;
   a.dsum = dsum;
+  a.out0 = static_cast<__nv_bfloat16*>(dv);
+  a.out1 = static_cast<__nv_bfloat16*>(dk);
   a.status = status;
   a.N = p.N;
   a.Np = Np;
   a.rs = p.row_stride;
   a.H = p.H;
-  a.nq = p.nq;
-  a.n_items = p.H * p.nq;
+  a.nq = nt;
+  a.n_items = p.H * nt;
+  a.nk_fine = p.nk;
+  a.k_rows_per_tile = p.block_k == 64 ? 2 : 1;
+  a.list_shift = p.block == 64 ? 1 : 0;
   a.scale = p.scale;
   a.scale_log2 = p.scale * 1.4426950408889634f;
   a.timeout_ns = timeout_ns;
-  BwdParams pq = a, pk = a;
-  pq.ptr = row_ptr;
-  pq.idx = col_idx;
-  pq.out0 = static_cast<__nv_bfloat16*>(dq);
-  pk.ptr = col_ptr_t;
-  pk.idx = row_idx_t;
-  pk.out0 = static_cast<__nv_bfloat16*>(dv);
-  pk.out1 = static_cast<__nv_bfloat16*>(dk);
-  if (kFusedBwd)
-    return p.d == 64 ? launch_bwd_fused<64>(p, tm, pk, dq_acc, static_cast<__nv_bfloat16*>(dq), sms, stream)
-                     : launch_bwd_fused<128>(p, tm, pk, dq_acc, static_cast<__nv_bfloat16*>(dq), sms, stream);
-  return p.d == 64 ? launch_bwd_d<64>(p, tm, pq, pk, sms, stream) : launch_bwd_d<128>(p, tm, pq, pk, sms, stream);
+  __nv_bfloat16* dqb = static_cast<__nv_bfloat16*>(dq);
+  const bool sub = p.block == 64 || p.block_k == 64;
+  if (p.d == 64)
+    return sub ? launch_bwd_fused<64, true>(p, tm, a, dq_acc, dqb, sms, stream)
+               : launch_bwd_fused<64, false>(p, tm, a, dq_acc, dqb, sms, stream);
+  return sub ? launch_bwd_fused<128, true>(p, tm, a, dq_acc, dqb, sms, stream)
+             : launch_bwd_fused<128, false>(p, tm, a, dq_acc, dqb, sms, stream);
 }
 
 }  // namespace ut

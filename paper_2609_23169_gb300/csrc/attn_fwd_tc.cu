@@ -19,6 +19,11 @@
 //               pairs into a TMEM P buffer, and finally normalises O and
 //               writes O (bf16) and LSE (fp32, natural log).
 // TMEM columns: S0 [0,128), S1 [128,256), O [256,256+D), P0 [384,448), P1 [448,512).
+// Blocks of 64 rows (b_q or b_kv) are served by the same 128 x 128 tiles: an
+// item's fine key-block lists are merged into 128-row key tiles with a mask of
+// the listed 64 x 64 sub-blocks (TileList), and the softmax sets the scores of
+// unlisted sub-blocks to -inf.  Rows that see no key end with O = 0 and
+// LSE = -inf.
 // Every wait is bounded; on expiry the kernel records UT_ERR_TIMEOUT,
 // drains its own copies and MMAs, frees TMEM and returns.
 #include "common.cuh"
@@ -51,20 +56,23 @@ struct FwdSmem {
 };
 
 struct FwdParams {
-  const int32_t* row_ptr;
+  const int32_t* row_ptr;   // fine lists: nq_fine rows per head
   const int32_t* col_idx;
+  int nq_fine;              // query blocks per head in the lists
+  int q_rows_per_tile;      // 1 (b_q = 128) or 2 (b_q = 64)
+  int list_shift;           // 0 (b_kv = 128) or 1 (b_kv = 64)
   __nv_bfloat16* o;
   float* lse;
   int32_t* status;
   int64_t N;
   int64_t rs;  // elements between tokens
-  int H, nq;
+  int H, nq;         // nq: 128-row query tiles per head
   int n_items;
   float scale_log2;  // softmax scale * log2(e)
   uint64_t timeout_ns;
 };
 
-template <int D>
+template <int D, bool kSub>
 __global__ void __launch_bounds__(kFwdThreads, 1)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                        const __grid_constant__ CUtensorMap tm_v, const FwdParams prm) {
@@ -128,7 +136,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int h = w / prm.nq, i = w % prm.nq;
-        const int beg = prm.row_ptr[w], L = prm.row_ptr[w + 1] - beg;
+        TileList<kSub> tl;
+        tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
+        const int L = tl.count();
         if (L <= 0) continue;
         if (is_k) {
           if (!(ok = mbar_wait(&sm.q_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -138,7 +148,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           ++qi;
         }
         for (int t = 0; t < L; ++t, ++kv) {
-          const int j = prm.col_idx[beg + t];
+          int j;
+          uint32_t bits;
+          tl.next(j, bits);
           const uint32_t st = kv % kStages, n = kv / kStages;
           if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
           mbar_expect_tx(&full[st], FwdSmem<D>::kKVBytes);
@@ -166,7 +178,10 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       uint32_t qi = 0, oi = 0, kv0 = 0, sc0 = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-        const int L = prm.row_ptr[w + 1] - prm.row_ptr[w];
+        TileList<kSub> tl;
+        tl.init(prm.row_ptr, prm.col_idx, w / prm.nq, w % prm.nq, prm.nq_fine, prm.q_rows_per_tile,
+                prm.list_shift);
+        const int L = tl.count();
         if (L <= 0) continue;
         if (!(ok = warp_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         // S runs two key blocks ahead of P V: S_{u+2} goes into the S buffer
@@ -228,9 +243,12 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     const float c = prm.scale_log2;
     uint32_t sc0 = 0;
     bool ok = true;
+    const uint32_t rh = row >> 6;  // which 64-row half of the query tile
     for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
       const int h = w / prm.nq, i = w % prm.nq;
-      const int beg = prm.row_ptr[w], L = prm.row_ptr[w + 1] - beg;
+      TileList<kSub> tl;
+      tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
+      const int L = tl.count();
       const int64_t grow = (int64_t)i * kBM + row;
       const bool row_ok = grow < prm.N;
       __nv_bfloat16* orow = prm.o + grow * prm.rs + (int64_t)h * D;
@@ -242,8 +260,13 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         continue;
       }
       float m_used = 0.f, l = 0.f;
-      int j_cur = prm.col_idx[beg];
+      int j_next = 0;
+      uint32_t bits_next = 0;
+      if (L > 0) tl.next(j_next, bits_next);
       for (int t = 0; t < L; ++t) {
+        const int j = j_next;
+        const uint32_t bits = bits_next;
+        if (t + 1 < L) tl.next(j_next, bits_next);  // the next tile's index, fetched a tile ahead
         const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
         if (!(ok = warp_wait(&sm.s_full[sb], ns & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
@@ -259,14 +282,24 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         float s[kBN];
 #pragma unroll
         for (int x = 0; x < kBN; ++x) s[x] = __uint_as_float(r[x]);
-        // ragged last key block: columns past N do not exist
-        const int j = j_cur;
-        if (t + 1 < L) j_cur = prm.col_idx[beg + t + 1];  // prefetch the next block index
+        // ragged last key block: columns past N do not exist; 64-column
+        // halves of the tile not listed for this row's half are masked
         const int64_t nv = prm.N - (int64_t)j * kBN;
+        const uint32_t cols = kSub ? (bits >> (2 * rh)) & 3u : 3u;
         if (nv < kBN) {
 #pragma unroll
           for (int x = 0; x < kBN; ++x)
             if (x >= nv) s[x] = -INFINITY;
+        }
+        if (kSub) {  // a masked half is the same for the whole warp (rh is per warp)
+          if (!(cols & 1u)) {
+#pragma unroll
+            for (int x = 0; x < kBN / 2; ++x) s[x] = -INFINITY;
+          }
+          if (!(cols & 2u)) {
+#pragma unroll
+            for (int x = kBN / 2; x < kBN; ++x) s[x] = -INFINITY;
+          }
         }
         // row maximum as a tree (8 independent chains) rather than one long chain
         float m8[8];
@@ -276,7 +309,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         for (int x = 8; x < kBN; ++x) m8[x & 7] = fmaxf(m8[x & 7], s[x]);
         float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
                          fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-        mx *= c;
+        // a row may see nothing in this tile: keep the reference maximum
+        // finite so that exp2(-inf - m) stays 0 (not NaN)
+        mx = kSub ? fmaxf(mx * c, -1e30f) : mx * c;
         if (t == 0) {
           m_used = mx;
         } else {
@@ -307,11 +342,19 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         uint32_t pk[kBN / 2];
         float l8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int x = 0; x < kBN; x += 2) {
-          const float p0 = ex2_approx(fmaf(s[x], c, -m_used));
-          const float p1 = ex2_approx(fmaf(s[x + 1], c, -m_used));
-          l8[(x >> 1) & 7] += p0 + p1;
-          pk[x / 2] = pack_bf16x2(p0, p1);
+        for (int hc = 0; hc < 2; ++hc) {
+          if (kSub && !((cols >> hc) & 1u)) {  // a masked half: P = 0 without the exponentials
+#pragma unroll
+            for (int x = hc * (kBN / 2); x < (hc + 1) * (kBN / 2); x += 2) pk[x / 2] = 0u;
+            continue;
+          }
+#pragma unroll
+          for (int x = hc * (kBN / 2); x < (hc + 1) * (kBN / 2); x += 2) {
+            const float p0 = ex2_approx(fmaf(s[x], c, -m_used));
+            const float p1 = ex2_approx(fmaf(s[x + 1], c, -m_used));
+            l8[(x >> 1) & 7] += p0 + p1;
+            pk[x / 2] = pack_bf16x2(p0, p1);
+          }
         }
         l += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
         // the TMEM P buffer is free once the P V MMA of its previous use finished
@@ -329,7 +372,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       const uint32_t last = sc0 + L - 1;
       if (!(ok = warp_wait(&sm.pv_done[last & 1], (last >> 1) & 1, abort_flag, prm.status, prm.timeout_ns))) break;
       tc_fence_after();
-      const float inv = 1.0f / l;
+      const float inv = (!kSub || l > 0.f) ? 1.0f / l : 0.f;  // a row that saw no key: O = 0, LSE = -inf
 #pragma unroll
       for (int g = 0; g < D / 32; ++g) {
         uint32_t r[32];
@@ -350,7 +393,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.o_empty);
-      if (row_ok) prm.lse[(int64_t)h * prm.N + grow] = (m_used + log2f(l)) * 0.69314718055994531f;
+      if (row_ok)
+        prm.lse[(int64_t)h * prm.N + grow] =
+            (!kSub || l > 0.f) ? (m_used + log2f(l)) * 0.69314718055994531f : -INFINITY;
       sc0 += L;
     }
   }
@@ -363,20 +408,22 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 
 static_assert(sizeof(FwdSmem<128>) + 1024 <= 232448, "forward shared layout exceeds the per-block limit");
 
-template <int D>
+template <int D, bool kSub>
 static cudaError_t launch_d(const AttnProblem& p, const CUtensorMap& tq, const CUtensorMap& tk,
                             const CUtensorMap& tv, const FwdParams& prm, int grid, cudaStream_t stream) {
   const size_t smem = sizeof(FwdSmem<D>) + 1024;
-  cudaError_t e = cudaFuncSetAttribute(attn_fwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e =
+      cudaFuncSetAttribute(attn_fwd_tc_kernel<D, kSub>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  attn_fwd_tc_kernel<D><<<grid, kFwdThreads, smem, stream>>>(tq, tk, tv, prm);
+  attn_fwd_tc_kernel<D, kSub><<<grid, kFwdThreads, smem, stream>>>(tq, tk, tv, prm);
   return cudaGetLastError();
 }
 
 cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* k, const void* v,
                                const int32_t* row_ptr, const int32_t* col_idx, void* o, float* lse, int32_t* status,
                                uint64_t timeout_ns, int sms, cudaStream_t stream) {
-  const int n_items = p.H * p.nq;
+  const int nt = (int)((p.N + kBM - 1) / kBM);  // 128-row tiles
+  const int n_items = p.H * nt;
   if (n_items == 0) return cudaSuccess;
   CUtensorMap tq, tk, tv;
   const uint64_t inner = (uint64_t)p.H * p.d;
@@ -394,12 +441,19 @@ cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* 
   prm.N = p.N;
   prm.rs = p.row_stride;
   prm.H = p.H;
-  prm.nq = p.nq;
+  prm.nq = nt;
+  prm.nq_fine = p.nq;
+  prm.q_rows_per_tile = p.block == 64 ? 2 : 1;
+  prm.list_shift = p.block_k == 64 ? 1 : 0;
   prm.n_items = n_items;
   prm.scale_log2 = p.scale * 1.4426950408889634f;
   prm.timeout_ns = timeout_ns;
   const int grid = n_items < sms ? n_items : sms;
-  return p.d == 64 ? launch_d<64>(p, tq, tk, tv, prm, grid, stream) : launch_d<128>(p, tq, tk, tv, prm, grid, stream);
+  const bool sub = p.block == 64 || p.block_k == 64;
+  if (p.d == 64)
+    return sub ? launch_d<64, true>(p, tq, tk, tv, prm, grid, stream) : launch_d<64, false>(p, tq, tk, tv, prm, grid, stream);
+  return sub ? launch_d<128, true>(p, tq, tk, tv, prm, grid, stream)
+             : launch_d<128, false>(p, tq, tk, tv, prm, grid, stream);
 }
 
 }  // namespace ut

@@ -1,8 +1,9 @@
 // Block mask M_c as key-block lists (Sec. 3.3).
 //
 // Top-K mode:
-//   block_pool_kernel    pool(Q), pool(K): fp32 mean over the valid rows of
-//                        each block, every head at once (one CTA per block).
+//   block_pool_kernel    pool(Q) over blocks of b_q rows, pool(K) over blocks
+//                        of b_kv rows: fp32 mean over the valid rows of each
+//                        block, every head at once (one CTA per block).
 //   score_select_kernel  S_c[i, :] = pool(Q)_i . pool(K)_j in fp32 for R query
 //                        blocks of one head, then per row an exact radix
 //                        select of the K_rho-th largest score (4 passes of 8
@@ -47,14 +48,20 @@ struct Vec8<float> {
   }
 };
 
-// grid (nq, 2): blockIdx.y selects Q (0) or K (1).  out: [2][H][nq][d].
+// grid (max(nq, nk), 2): blockIdx.y selects Q (0, blocks of bq rows) or K (1,
+// blocks of bk rows).  out: pooled Q [H][nq][d], then pooled K [H][nk][d].
 template <typename T>
 __global__ void __launch_bounds__(kPoolThreads) block_pool_kernel(const T* __restrict__ q, const T* __restrict__ k,
                                                                   int64_t N, int H, int d, int64_t row_stride,
-                                                                  int block, int nq, float* __restrict__ out) {
+                                                                  int bq, int nq, int bk, int nk,
+                                                                  float* __restrict__ out) {
   constexpr int E = Vec8<T>::kElems;
-  const T* x = blockIdx.y == 0 ? q : k;
+  const bool is_k = blockIdx.y == 1;
+  const T* x = is_k ? k : q;
+  const int block = is_k ? bk : bq, nb = is_k ? nk : nq;
   const int i = blockIdx.x;
+  if (i >= nb) return;
+  float* base = is_k ? out + (size_t)H * nq * d : out;
   const int64_t r0 = (int64_t)i * block;
   const int64_t r1 = min(N, r0 + block);
   const int cols = H * d;
@@ -71,7 +78,7 @@ __global__ void __launch_bounds__(kPoolThreads) block_pool_kernel(const T* __res
     }
     const int c0 = ch * E;
     const int h = c0 / d, e0 = c0 % d;
-    float* dst = out + (((int64_t)blockIdx.y * H + h) * nq + i) * d + e0;
+    float* dst = base + ((int64_t)h * nb + i) * d + e0;
 #pragma unroll
     for (int e = 0; e < E; ++e) dst[e] = __fdiv_rn(acc[e], (float)(r1 - r0));
     (void)inv_cnt;
@@ -85,22 +92,23 @@ UT_DEV uint32_t order_key(float s) {
 }
 
 // grid (H, ceil(nq / R)); dynamic smem: R*d + R*nk floats + 8 warps * 256 ints.
+// Rows are query blocks (nq per head), columns key blocks (nk).
 __global__ void __launch_bounds__(kSelThreads) score_select_kernel(const float* __restrict__ pooled, int H, int d,
-                                                                   int nq, int R, int k_rho,
+                                                                   int nq, int nk, int R, int k_rho,
                                                                    int32_t* __restrict__ col_idx,
                                                                    uint8_t* __restrict__ bitmap) {
   extern __shared__ float smem[];
   float* pq = smem;                       // [R][d]
-  float* sc = smem + R * d;               // [R][nq]
-  uint32_t* hist = reinterpret_cast<uint32_t*>(sc + R * nq);  // [8][256]
+  float* sc = smem + R * d;               // [R][nk]
+  uint32_t* hist = reinterpret_cast<uint32_t*>(sc + R * nk);  // [8][256]
   const int h = blockIdx.x;
   const int i0 = blockIdx.y * R;
   const int rows = min(R, nq - i0);
   const float* PQ = pooled + ((int64_t)h * nq) * d;
-  const float* PK = pooled + ((int64_t)(H + h) * nq) * d;
+  const float* PK = pooled + (int64_t)H * nq * d + ((int64_t)h * nk) * d;
   for (int t = threadIdx.x; t < rows * d; t += kSelThreads) pq[t] = PQ[(int64_t)i0 * d + t];
   __syncthreads();
-  for (int j = threadIdx.x; j < nq; j += kSelThreads) {
+  for (int j = threadIdx.x; j < nk; j += kSelThreads) {
     float acc[kSelMaxRows];
 #pragma unroll
     for (int r = 0; r < kSelMaxRows; ++r) acc[r] = 0.f;
@@ -119,21 +127,21 @@ __global__ void __launch_bounds__(kSelThreads) score_select_kernel(const float* 
     }
 #pragma unroll
     for (int r = 0; r < kSelMaxRows; ++r)
-      if (r < rows) sc[r * nq + j] = acc[r];
+      if (r < rows) sc[r * nk + j] = acc[r];
   }
   __syncthreads();
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   uint32_t* hw = hist + w * 256;
   const uint32_t lt_mask = (1u << lane) - 1u;
   for (int r = w; r < rows; r += kSelThreads / 32) {
-    const float* srow = sc + r * nq;
+    const float* srow = sc + r * nk;
     uint32_t prefix = 0, pmask = 0;
     int k = k_rho;  // rank still to find among keys matching the prefix
     for (int pass = 3; pass >= 0; --pass) {
       const int shift = pass * 8;
       for (int b = lane; b < 256; b += 32) hw[b] = 0;
       __syncwarp();
-      for (int j = lane; j < nq; j += 32) {
+      for (int j = lane; j < nk; j += 32) {
         uint32_t u = order_key(srow[j]);
         if ((u & pmask) == prefix) atomicAdd(&hw[(u >> shift) & 255u], 1u);
       }
@@ -177,12 +185,12 @@ __global__ void __launch_bounds__(kSelThreads) score_select_kernel(const float* 
     // prefix = the K_rho-th largest key; take all larger keys and the first k equal ones.
     const int row = h * nq + i0 + r;
     int32_t* out = col_idx + (int64_t)row * k_rho;
-    uint8_t* brow = bitmap + (int64_t)row * nq;
+    uint8_t* brow = bitmap + (int64_t)row * nk;
     int n_sel = 0, n_eq = 0;
-    for (int j0 = 0; j0 < nq; j0 += 32) {
+    for (int j0 = 0; j0 < nk; j0 += 32) {
       const int j = j0 + lane;
-      uint32_t u = j < nq ? order_key(srow[j]) : 0u;
-      const bool valid = j < nq;
+      uint32_t u = j < nk ? order_key(srow[j]) : 0u;
+      const bool valid = j < nk;
       const bool gt = valid && u > prefix;
       const bool eq = valid && u == prefix;
       const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
@@ -279,18 +287,18 @@ __global__ void bitmap_fill_kernel(const uint8_t* __restrict__ bm, int H, int nq
 }
 
 // ----------------------------------------------------------------- launchers
-static int select_rows(int nq) {
-  int r = (64 * 1024) / (nq * 4);
+static int select_rows(int nk) {
+  int r = (64 * 1024) / (nk * 4);
   r = r < 1 ? 1 : r;
   return r > kSelMaxRows ? kSelMaxRows : r;
 }
 
 size_t block_mask_ws(const MaskProblem& p, int mode) {
-  const size_t H = p.H, nq = p.nq, d = p.d;
-  size_t counts = (H * nq + 1) * sizeof(int32_t);
+  const size_t H = p.H, nq = p.nq, nk = p.nk, d = p.d;
+  size_t counts = (H * (nq > nk ? nq : nk) + 1) * sizeof(int32_t);
   if (mode == UT_MASK_BITMAP) return counts;
-  size_t pooled = 2 * H * nq * d * sizeof(float);
-  size_t bitmap = H * nq * nq;
+  size_t pooled = H * (nq + nk) * d * sizeof(float);
+  size_t bitmap = H * nq * nk;
   return pooled + ((bitmap + 255) / 256) * 256 + counts;
 }
 
@@ -310,29 +318,29 @@ cudaError_t launch_block_mask_topk(const MaskProblem& p, const void* q, const vo
                                    int32_t* col_idx, int32_t* col_ptr_t, int32_t* row_idx_t, int64_t col_cap,
                                    void* ws, int32_t* status, int sms, cudaStream_t stream) {
   (void)sms;
-  const int H = p.H, nq = p.nq, d = p.d;
+  const int H = p.H, nq = p.nq, nk = p.nk, d = p.d;
   float* pooled = static_cast<float*>(ws);
-  uint8_t* bitmap = reinterpret_cast<uint8_t*>(pooled + (size_t)2 * H * nq * d);
-  size_t bm_bytes = (((size_t)H * nq * nq + 255) / 256) * 256;
+  uint8_t* bitmap = reinterpret_cast<uint8_t*>(pooled + (size_t)H * (nq + nk) * d);
+  size_t bm_bytes = (((size_t)H * nq * nk + 255) / 256) * 256;
   int32_t* counts = reinterpret_cast<int32_t*>(bitmap + bm_bytes);
-  dim3 pg(nq, 2);
+  dim3 pg(nq > nk ? nq : nk, 2);
   if (p.dtype == UT_BF16)
     block_pool_kernel<__nv_bfloat16><<<pg, kPoolThreads, 0, stream>>>(
         static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), p.N, H, d, p.row_stride, p.block,
-        nq, pooled);
+        nq, p.block_k, nk, pooled);
   else
     block_pool_kernel<float><<<pg, kPoolThreads, 0, stream>>>(static_cast<const float*>(q),
                                                               static_cast<const float*>(k), p.N, H, d, p.row_stride,
-                                                              p.block, nq, pooled);
-  const int R = select_rows(nq);
-  size_t smem = ((size_t)R * d + (size_t)R * nq) * sizeof(float) + 8 * 256 * sizeof(uint32_t);
+                                                              p.block, nq, p.block_k, nk, pooled);
+  const int R = select_rows(nk);
+  size_t smem = ((size_t)R * d + (size_t)R * nk) * sizeof(float) + 8 * 256 * sizeof(uint32_t);
   cudaError_t e = cudaFuncSetAttribute(score_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 sg(H, (nq + R - 1) / R);
-  score_select_kernel<<<sg, kSelThreads, smem, stream>>>(pooled, H, d, nq, R, k_rho, col_idx, bitmap);
+  score_select_kernel<<<sg, kSelThreads, smem, stream>>>(pooled, H, d, nq, nk, R, k_rho, col_idx, bitmap);
   fill_uniform_rowptr_kernel<<<(H * nq + 1 + 255) / 256, 256, 0, stream>>>(row_ptr, H * nq, k_rho);
   if (col_ptr_t && row_idx_t) {
-    e = csr_from_bitmap(bitmap, H, nq, nq, 1, col_ptr_t, row_idx_t, col_cap, counts, status, stream);
+    e = csr_from_bitmap(bitmap, H, nq, nk, 1, col_ptr_t, row_idx_t, col_cap, counts, status, stream);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
@@ -342,10 +350,10 @@ cudaError_t launch_block_mask_bitmap(const MaskProblem& p, const uint8_t* bitmap
                                      int32_t* col_ptr_t, int32_t* row_idx_t, int64_t col_cap, void* ws,
                                      int32_t* status, cudaStream_t stream) {
   int32_t* counts = static_cast<int32_t*>(ws);
-  cudaError_t e = csr_from_bitmap(bitmap, p.H, p.nq, p.nq, 0, row_ptr, col_idx, col_cap, counts, status, stream);
+  cudaError_t e = csr_from_bitmap(bitmap, p.H, p.nq, p.nk, 0, row_ptr, col_idx, col_cap, counts, status, stream);
   if (e != cudaSuccess) return e;
   if (col_ptr_t && row_idx_t)
-    e = csr_from_bitmap(bitmap, p.H, p.nq, p.nq, 1, col_ptr_t, row_idx_t, col_cap, counts, status, stream);
+    e = csr_from_bitmap(bitmap, p.H, p.nq, p.nk, 1, col_ptr_t, row_idx_t, col_cap, counts, status, stream);
   return e;
 }
 

@@ -187,6 +187,85 @@ UT_DEV void setmaxnreg_dec() {
   asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
 
+// ------------------------------------------------------------ tile lists
+// The tensor-core kernels work on 128-row tiles; the block lists may be at a
+// 64-row granularity on either side (b_q, b_kv in {64, 128}).  An item (one
+// 128-row tile of the listing side) then owns one or two fine list rows, and
+// a listed 64-row block falls in tile j >> 1.  TileList merges the item's
+// fine lists into ascending 128-row tiles and, per tile, a 2 x 2 mask of the
+// 64 x 64 sub-blocks that are listed:
+//   bit (2 * r + c): rows r * 64 .. r * 64 + 63 of the item's tile may see
+//   columns c * 64 .. c * 64 + 63 of the listed tile.
+// With 128-row blocks on both sides every listed tile has all four bits.
+template <bool kSub>  // kSub: 64-row blocks on at least one side
+struct TileList {
+  const int32_t* a;   // fine list of the item's first (or only) row block
+  const int32_t* b;   // fine list of its second 64-row block, if any
+  int na, nb, pa, pb;
+  int shift;          // 1 when the listed blocks have 64 rows
+  bool split;         // the item holds two 64-row blocks (a: rows 0-63, b: rows 64-127)
+
+  // item = (row-block tile t of head h); ptr/idx the fine lists with nfine
+  // rows per head; rows_per_tile = 2 for 64-row blocks on the listing side.
+  UT_DEV void init(const int32_t* ptr, const int32_t* idx, int h, int t, int nfine, int rows_per_tile,
+                   int list_shift) {
+    const int r0 = kSub ? t * rows_per_tile : t;
+    const int64_t base = (int64_t)h * nfine;
+    const int s0 = ptr[base + r0];
+    a = idx + s0;
+    na = ptr[base + r0 + 1] - s0;
+    pa = pb = 0;
+    b = a;
+    nb = 0;
+    split = false;
+    shift = 0;
+    if (kSub) {
+      split = rows_per_tile == 2;
+      shift = list_shift;
+      if (split && r0 + 1 < nfine) {
+        const int s1 = ptr[base + r0 + 1];
+        b = idx + s1;
+        nb = ptr[base + r0 + 2] - s1;
+      }
+    }
+  }
+  // next listed tile and its sub-block mask; false at the end
+  UT_DEV bool next(int& tile, uint32_t& bits) {
+    if (!kSub) {  // 128-row blocks on both sides: the list itself, every sub-block
+      if (pa >= na) return false;
+      tile = a[pa++];
+      bits = 15u;
+      return true;
+    }
+    const int ta = pa < na ? (a[pa] >> shift) : 0x7fffffff;
+    const int tb = pb < nb ? (b[pb] >> shift) : 0x7fffffff;
+    tile = ta < tb ? ta : tb;
+    if (tile == 0x7fffffff) return false;
+    const uint32_t rows_a = split ? 1u : 3u;
+    bits = 0;
+    while (pa < na && (a[pa] >> shift) == tile) {
+      const uint32_t cols = shift ? (1u << (a[pa] & 1)) : 3u;
+      bits |= ((rows_a & 1u) ? cols : 0u) | ((rows_a & 2u) ? cols << 2 : 0u);
+      ++pa;
+    }
+    while (pb < nb && (b[pb] >> shift) == tile) {
+      const uint32_t cols = shift ? (1u << (b[pb] & 1)) : 3u;
+      bits |= cols << 2;
+      ++pb;
+    }
+    return true;
+  }
+  // number of listed tiles (walks a copy)
+  UT_DEV int count() const {
+    if (!kSub) return na - pa;
+    TileList c = *this;
+    int n = 0, t;
+    uint32_t m;
+    while (c.next(t, m)) ++n;
+    return n;
+  }
+};
+
 // ---------------------------------------------------------------- tcgen05
 UT_DEV void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),

@@ -36,7 +36,9 @@ struct MaskProblem {
   int64_t N;
   int H, d, block, dtype;
   int64_t row_stride;
-  int nq;  // = nk
+  int nq;       // query blocks of `block` rows
+  int block_k;  // rows per key block
+  int nk;       // key blocks
 };
 size_t block_mask_ws(const MaskProblem& p, int mode);
 cudaError_t launch_block_mask_topk(const MaskProblem& p, const void* q, const void* k, int k_rho, int32_t* row_ptr,
@@ -51,8 +53,10 @@ struct AttnProblem {
   int64_t N;
   int H, d, block, dtype;
   int64_t row_stride;
-  int nq;
+  int nq;        // query blocks of `block` rows (rows of the CSR lists per head)
   float scale;
+  int block_k;   // rows per key block
+  int nk;        // key blocks (rows of the transposed lists per head)
 };
 
 // attn_simt.cu (fp32 path and the generic CUDA-core backward)
@@ -70,7 +74,7 @@ cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* 
                                const int32_t* row_ptr, const int32_t* col_idx, void* o, float* lse, int32_t* status,
                                uint64_t timeout_ns, int sms, cudaStream_t stream);
 
-// attn_bwd_tc.cu (bf16 tcgen05 backward: preprocess, dK/dV, dQ)
+// attn_bwd_tc.cu (bf16 tcgen05 backward: preprocess, fused dK/dV/dQ, dQ finalize)
 size_t attn_bwd_tc_ws(const AttnProblem& p);
 cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* k, const void* v, const void* o,
                                const float* lse, const void* dout, const int32_t* row_ptr, const int32_t* col_idx,

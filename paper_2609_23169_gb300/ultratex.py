@@ -37,7 +37,8 @@ class UtError(RuntimeError):
 
 class AttnShape(ctypes.Structure):
     _fields_ = [("n_tokens", ctypes.c_int64), ("n_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
-                ("block", ctypes.c_int32), ("dtype", ctypes.c_int32), ("row_stride", ctypes.c_int64)]
+                ("block", ctypes.c_int32), ("dtype", ctypes.c_int32), ("row_stride", ctypes.c_int64),
+                ("block_k", ctypes.c_int32)]
 
 
 class Rope(ctypes.Structure):
@@ -147,11 +148,12 @@ def _dtype_code(t: torch.Tensor) -> int:
     raise TypeError(f"unsupported dtype {t.dtype}")
 
 
-def attn_shape(x: torch.Tensor, block: int) -> AttnShape:
-    """Shape of a token-major [N, H, d] tensor (rows may be padded: stride(0) >= H*d)."""
+def attn_shape(x: torch.Tensor, block: int, block_k: int = 0) -> AttnShape:
+    """Shape of a token-major [N, H, d] tensor (rows may be padded: stride(0) >= H*d);
+    query blocks of `block` rows, key blocks of `block_k` rows (0: same)."""
     N, H, d = x.shape
     assert x.stride(2) == 1 and x.stride(1) == d, "heads must be contiguous within a token row"
-    return AttnShape(N, H, d, block, _dtype_code(x), x.stride(0))
+    return AttnShape(N, H, d, block, _dtype_code(x), x.stride(0), block_k)
 
 
 def status_word(device=None) -> torch.Tensor:
@@ -304,15 +306,16 @@ def ut_block_mask(shape: AttnShape, mode: int, q: Optional[torch.Tensor] = None,
                   out: Optional[tuple] = None):
     """Key-block lists.  Returns (row_ptr, col_idx, col_ptr_t, row_idx_t) (the last two None if not asked)."""
     nq = -(-shape.n_tokens // shape.block)
+    nk = -(-shape.n_tokens // (shape.block_k or shape.block))
     H = shape.n_heads
     dev = (q if q is not None else bitmap).device
     L = lib()
     if col_cap is None:
-        col_cap = H * nq * (ut_topk_count(rho, nq) if mode == UT_MASK_TOPK else nq)
+        col_cap = H * nq * (ut_topk_count(rho, nk) if mode == UT_MASK_TOPK else nk)
     if out is None:
         row_ptr = torch.empty(H * nq + 1, dtype=torch.int32, device=dev)
         col_idx = torch.empty(max(col_cap, 1), dtype=torch.int32, device=dev)
-        col_ptr = torch.empty(H * nq + 1, dtype=torch.int32, device=dev) if with_transpose else None
+        col_ptr = torch.empty(H * nk + 1, dtype=torch.int32, device=dev) if with_transpose else None
         row_idx = torch.empty(max(col_cap, 1), dtype=torch.int32, device=dev) if with_transpose else None
     else:
         row_ptr, col_idx, col_ptr, row_idx = out
@@ -329,9 +332,10 @@ def ut_block_mask(shape: AttnShape, mode: int, q: Optional[torch.Tensor] = None,
 
 def ut_bsattn_fwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, row_ptr: torch.Tensor, col_idx: torch.Tensor,
                   block: int, softmax_scale: Optional[float] = None, o: Optional[torch.Tensor] = None,
-                  lse: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None):
-    """Block-sparse attention forward.  Returns (O [N,H,d], LSE [H,N] fp32)."""
-    shape = attn_shape(q, block)
+                  lse: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None, block_k: int = 0):
+    """Block-sparse attention forward (query blocks of `block` rows, key blocks of
+    `block_k` rows, 0: same).  Returns (O [N,H,d], LSE [H,N] fp32)."""
+    shape = attn_shape(q, block, block_k)
     N, H, d = q.shape
     scale = d ** -0.5 if softmax_scale is None else float(softmax_scale)
     if o is None:
@@ -345,9 +349,10 @@ def ut_bsattn_fwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, row_ptr: to
 
 
 def ut_bsattn_bwd(q, k, v, o, lse, dout, row_ptr, col_idx, col_ptr_t, row_idx_t, block: int,
-                  softmax_scale: Optional[float] = None, dq=None, dk=None, dv=None, ws=None, status=None):
+                  softmax_scale: Optional[float] = None, dq=None, dk=None, dv=None, ws=None, status=None,
+                  block_k: int = 0):
     """Gradient of ut_bsattn_fwd.  Returns (dQ, dK, dV)."""
-    shape = attn_shape(q, block)
+    shape = attn_shape(q, block, block_k)
     d = q.shape[2]
     scale = d ** -0.5 if softmax_scale is None else float(softmax_scale)
     dq = torch.empty_like(q) if dq is None else dq

@@ -54,8 +54,20 @@ def test_argument_errors_are_caught_on_host(L):
         == u.UT_ERR_UNSUPPORTED
     assert L.ut_bsattn_fwd(S(_shape(u, dtype=7)), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
         == u.UT_ERR_INVALID_ARG
-    assert L.ut_bsattn_fwd(S(_shape(u, dtype=0, b=64)), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None,
+    assert L.ut_bsattn_fwd(S(_shape(u, dtype=0, b=32)), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None,
                            None) == u.UT_ERR_UNSUPPORTED
+    # unequal blocks: bf16 only, each 64 or 128
+    sh = _shape(u, dtype=1, b=64)
+    sh.block_k = 128
+    assert L.ut_bsattn_fwd(S(sh), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
+        == u.UT_ERR_UNSUPPORTED
+    sh = _shape(u, dtype=0, b=128)
+    sh.block_k = 32
+    assert L.ut_bsattn_fwd(S(sh), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
+        == u.UT_ERR_UNSUPPORTED
+    sh.block_k = -1
+    assert L.ut_bsattn_fwd(S(sh), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
+        == u.UT_ERR_INVALID_ARG
     # bad row stride, null pointers, bad scale, misalignment
     assert L.ut_bsattn_fwd(S(_shape(u, rs=100)), bogus, bogus, bogus, bogus, bogus, 0.1, bogus, bogus, None, None) \
         == u.UT_ERR_INVALID_ARG
