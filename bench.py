@@ -556,10 +556,6 @@ def run_sweep(args):
             for rho in sorted(SWEEP_RHO, reverse=True):
                 w = sweep2048(fg, rho, block)
                 line = {"sweep": True, "workload": w.name, "fg": fg, "rho": rho, "block": block, "N": w.N}
-                if block != 128:
-                    line["unavailable"] = "bf16 block size 64 has no tensor-core kernel yet (UT_ERR_UNSUPPORTED)"
-                    print(json.dumps(line), flush=True)
-                    continue
                 hp = P.HotPath(w.T, w.heads, w.head_dim, block, torch.bfloat16, u.UT_MASK_TOPK, rho=rho, device=dev)
                 N = hp.step(mask, q, k, v, do)
                 torch.cuda.synchronize()

@@ -230,8 +230,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
           const int h = w / prm.nq, j = w % prm.nq;
           TileList<kSub> tl;
           tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
-          const int L = tl.count();
-          if (L <= 0) continue;
+          if (tl.empty()) continue;
           if (is_q) {
             if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             mbar_expect_tx(&sm.kv_full, 2 * TB);
@@ -241,10 +240,9 @@ __global__ void __launch_bounds__(kFuThreads, 1)
             }
             ++ki;
           }
-          for (int t = 0; t < L; ++t, ++qd) {
-            int i;
-            uint32_t bits;
-            tl.next(i, bits);
+          int i;
+          uint32_t bits;
+          for (; tl.next(i, bits); ++qd) {
             const uint32_t st = qd % nst, n = qd / nst;
             if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             mbar_expect_tx(&full[st], TB);
@@ -272,7 +270,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
           TileList<kSub> tl;
           tl.init(prm.ptr, prm.idx, w / prm.nq, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
-          const int L = tl.count();
+          const int L = tl.count_warp();
           if (L <= 0) continue;
           if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
           auto issue_st = [&](int t) -> bool {  // S^T_t = K Q_t^T into R0
@@ -371,7 +369,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
       const int h = w / prm.nq, j = w % prm.nq;
       TileList<kSub> tl;
       tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
-      const int L = tl.count();
+      const int L = tl.count_warp();
       const int64_t gk = (int64_t)j * kTile + krow;
       const bool row_ok = gk < prm.N;
       __nv_bfloat16* dv_row = prm.out0 + gk * prm.rs + (int64_t)h * D + half * HD;
@@ -523,7 +521,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
       const int h = w / prm.nq;
       TileList<kSub> tl;
       tl.init(prm.ptr, prm.idx, h, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
-      const int L = tl.count();
+      const int L = tl.count_warp();
       if (L <= 0) continue;
       for (int t = 0; t < L; ++t) {
         const uint32_t qd = qd0 + t;

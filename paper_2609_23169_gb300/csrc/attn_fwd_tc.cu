@@ -138,8 +138,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         const int h = w / prm.nq, i = w % prm.nq;
         TileList<kSub> tl;
         tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
-        const int L = tl.count();
-        if (L <= 0) continue;
+        if (tl.empty()) continue;
         if (is_k) {
           if (!(ok = mbar_wait(&sm.q_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
           mbar_expect_tx(&sm.q_full, FwdSmem<D>::kQBytes);
@@ -147,10 +146,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
             tma_load_2d(sm.q + c * kTileChunkBytes, &tm_q, &sm.q_full, h * D + c * 64, i * kBM, pol_q);
           ++qi;
         }
-        for (int t = 0; t < L; ++t, ++kv) {
-          int j;
-          uint32_t bits;
-          tl.next(j, bits);
+        int j;
+        uint32_t bits;
+        for (; tl.next(j, bits); ++kv) {
           const uint32_t st = kv % kStages, n = kv / kStages;
           if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
           mbar_expect_tx(&full[st], FwdSmem<D>::kKVBytes);
@@ -181,7 +179,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         TileList<kSub> tl;
         tl.init(prm.row_ptr, prm.col_idx, w / prm.nq, w % prm.nq, prm.nq_fine, prm.q_rows_per_tile,
                 prm.list_shift);
-        const int L = tl.count();
+        const int L = tl.count_warp();
         if (L <= 0) continue;
         if (!(ok = warp_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         // S runs two key blocks ahead of P V: S_{u+2} goes into the S buffer
@@ -248,7 +246,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       const int h = w / prm.nq, i = w % prm.nq;
       TileList<kSub> tl;
       tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
-      const int L = tl.count();
+      const int L = tl.count_warp();
       const int64_t grow = (int64_t)i * kBM + row;
       const bool row_ok = grow < prm.N;
       __nv_bfloat16* orow = prm.o + grow * prm.rs + (int64_t)h * D;

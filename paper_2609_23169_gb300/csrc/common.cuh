@@ -255,14 +255,40 @@ struct TileList {
     }
     return true;
   }
-  // number of listed tiles (walks a copy)
-  UT_DEV int count() const {
-    if (!kSub) return na - pa;
-    TileList c = *this;
-    int n = 0, t;
-    uint32_t m;
-    while (c.next(t, m)) ++n;
-    return n;
+  UT_DEV bool empty() const { return na == 0 && nb == 0; }
+
+  // number of listed tiles; the whole warp calls it (converged): the distinct
+  // tiles of each list are counted 32 entries at a time with ballots, and a
+  // tile listed by both lists is found by a binary search in the other one
+  UT_DEV int count_warp() const {
+    if (!kSub) return na;
+    const uint32_t lane = threadIdx.x & 31u;
+    int total = 0;
+    for (int which = 0; which < 2; ++which) {
+      const int32_t* x = which ? b : a;
+      const int nx = which ? nb : na;
+      const int32_t* y = which ? a : b;  // the other list (for shared tiles)
+      const int ny = which ? na : nb;
+      for (int i0 = 0; i0 < nx; i0 += 32) {
+        const int i = i0 + (int)lane;
+        bool fresh = false, shared = false;
+        if (i < nx) {
+          const int t = x[i] >> shift;
+          fresh = i == 0 || (x[i - 1] >> shift) != t;
+          if (fresh && which == 0 && ny > 0) {  // count a tile both lists hold once
+            int lo = 0, hi = ny;                // first y entry with (y >> shift) >= t
+            while (lo < hi) {
+              const int mid = (lo + hi) >> 1;
+              if ((y[mid] >> shift) < t) lo = mid + 1;
+              else hi = mid;
+            }
+            shared = lo < ny && (y[lo] >> shift) == t;
+          }
+        }
+        total += __popc(__ballot_sync(0xffffffffu, fresh)) - __popc(__ballot_sync(0xffffffffu, shared));
+      }
+    }
+    return total;
   }
 };
 
