@@ -231,27 +231,32 @@ def run_ours(args, rank, world, local_rank):
     value = flops_total / (ms_total * 1e-3) / 1e12
 
     # ---- e2e through host buffers: every step copies its canvas inputs from
-    # pinned host memory and its canvas results back; three streams overlap
-    # the copies of neighbouring steps with the compute of the current one
-    # (double-buffered device inputs and outputs).
+    # pinned host memory and its canvas results back.  The copies of
+    # neighbouring steps overlap the compute of the current one (three sets
+    # of device inputs and outputs); uploads and downloads share one
+    # copy stream, one direction at a time, because the host link moves less
+    # in total when both directions run at once.
     e2e = None
     if not args.no_e2e:
         pin_in = [x.pin_memory() for x in (torch.from_numpy(mask_np), q, k, v, do)]
+        NB = 3  # buffer sets: a step's outputs stay untouched until its download ends two steps later
         pin_out = [[torch.empty((w.T, w.heads, w.head_dim), dtype=torch.bfloat16).pin_memory() for _ in range(4)]
-                   for _ in range(2)]
+                   for _ in range(NB)]
         h2d = sum(x.numel() * x.element_size() for x in pin_in)
         d2h = sum(x.numel() * x.element_size() for x in pin_out[0])
-        dev_in = [[mask, tq, tk, tv, tdo], [torch.empty_like(x) for x in (mask, tq, tk, tv, tdo)]]
-        paths = [hp, P.HotPath(w.T, w.heads, w.head_dim, w.block, torch.bfloat16, u.UT_MASK_TOPK, rho=w.rho,
-                               device=dev)]
-        s_up, s_cmp, s_dn = torch.cuda.Stream(dev), torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        dev_in = [[mask, tq, tk, tv, tdo]] + [[torch.empty_like(x) for x in (mask, tq, tk, tv, tdo)]
+                                              for _ in range(NB - 1)]
+        paths = [hp] + [P.HotPath(w.T, w.heads, w.head_dim, w.block, torch.bfloat16, u.UT_MASK_TOPK, rho=w.rho,
+                                  device=dev) for _ in range(NB - 1)]
+        s_cmp = torch.cuda.Stream(dev)
+        s_up = s_dn = torch.cuda.Stream(dev)   # one copy stream for both directions
         ev = lambda: torch.cuda.Event(enable_timing=False)  # noqa: E731
-        in_ready = [ev(), ev()]
-        in_free = [None, None]
-        out_free = [None, None]
+        in_ready = [ev() for _ in range(NB)]
+        in_free = [None] * NB
+        out_free = [None] * NB
 
         def upload(k_):
-            b = k_ % 2
+            b = k_ % NB
             with torch.cuda.stream(s_up):
                 if in_free[b] is not None:
                     s_up.wait_event(in_free[b])
@@ -259,8 +264,8 @@ def run_ours(args, rank, world, local_rank):
                     dvc.copy_(hst, non_blocking=True)
                 in_ready[b].record(s_up)
 
-        def compute_and_download(k_):
-            b = k_ % 2
+        def compute(k_):
+            b = k_ % NB
             with torch.cuda.stream(s_cmp):
                 s_cmp.wait_event(in_ready[b])
                 if out_free[b] is not None:
@@ -270,8 +275,11 @@ def run_ours(args, rank, world, local_rank):
                 done = ev()
                 done.record(s_cmp)
                 in_free[b] = done
+
+        def download(k_):
+            b = k_ % NB
             with torch.cuda.stream(s_dn):
-                s_dn.wait_event(done)
+                s_dn.wait_event(in_free[b])
                 for hst, dvc in zip(pin_out[b], [paths[b].o_canvas] + paths[b].g_canvas):
                     hst.copy_(dvc, non_blocking=True)
                 fin = ev()
@@ -279,11 +287,17 @@ def run_ours(args, rank, world, local_rank):
                 out_free[b] = fin
 
         def run(n_steps):
+            # step k's results are downloaded while step k+1 computes, queued
+            # only after step k+1 has read its token count N (a 4-byte read
+            # that would otherwise wait behind a whole download)
             upload(0)
             for k_ in range(n_steps):
                 if k_ + 1 < n_steps:
                     upload(k_ + 1)
-                compute_and_download(k_)
+                compute(k_)
+                if k_ >= 1:
+                    download(k_ - 1)
+            download(n_steps - 1)
 
         run(2)
         torch.cuda.synchronize()
@@ -308,7 +322,8 @@ def run_ours(args, rank, world, local_rank):
             e_ms = float(t.item())
         e2e = {"value": round(world * f_step / (e_ms * 1e-3) / 1e12, 3), "unit": "TFLOP/s",
                "ms_per_step": round(e_ms, 3), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-               "pipeline": "3 streams (H2D | compute | D2H), double-buffered device inputs and outputs"}
+               "pipeline": "2 streams (copies in both directions, one at a time | compute), 3 sets of device "
+                           "inputs and outputs"}
 
     peaks, peak_src = load_peaks()
     # DRAM bytes per launch of each entry point from the last ncu capture of the

@@ -80,6 +80,12 @@ typedef struct {
 
 const char* ut_strerror(ut_status s);
 
+/* 1 if kernels on the current device can read and write `ptr` directly
+ * (device memory, or host memory mapped into the device's address space,
+ * such as pinned memory on systems with unified addressing); 0 otherwise,
+ * including on any error.  No device work is enqueued. */
+int32_t ut_device_accessible(const void* ptr);
+
 /* K_rho = max(1, floor(rho * n_k)) evaluated in double precision
  * (Sec. 3.3, the Top-K retention count). */
 int32_t ut_topk_count(double rho, int64_t n_k);
@@ -95,7 +101,10 @@ int32_t ut_topk_count(double rho, int64_t n_k);
  *   row_bytes bytes per token row (multiple of 16; pointers 16-byte aligned).
  *   capacity  rows available in each dst and in idx_out.
  *   idx_out   [capacity] int32: canvas position of compacted row n, ascending.
- *   n_out     one int32 (device): N = number of foreground tokens.
+ *   n_out     one int32 the kernels can address (device memory, or pinned host
+ *             memory where ut_device_accessible says so: the host then reads N
+ *             after an event instead of a copy that could queue behind other
+ *             transfers): N = number of foreground tokens.
  *   ws        workspace of ut_fg_compact_workspace_size(T) bytes.
  *   dev_status (may be NULL) receives UT_ERR_CAPACITY when N > capacity; rows
  *             beyond capacity are then not written (n_out still holds N).

@@ -227,6 +227,17 @@ ut_status ut_fg_scatter_rope(const int32_t* idx, int64_t n, int32_t n_tensors, c
                                   rope->prefix, rope->axes, rope->theta, mode, T, device_sms(), static_cast<cudaStream_t>(stream)));
 }
 
+int32_t ut_device_accessible(const void* ptr) {
+  if (!ptr) return 0;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+    (void)cudaGetLastError();  // not a CUDA-known pointer: clear the error
+    return 0;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return 1;
+  return a.type == cudaMemoryTypeHost && a.devicePointer == ptr ? 1 : 0;
+}
+
 ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int32_t channels,
                              int32_t dtype, float dt, int32_t* dev_status, void* stream) {
   if (n < 0 || T < 0 || n > T || channels <= 0) return UT_ERR_INVALID_ARG;

@@ -27,6 +27,12 @@ class HotPath:
         self.xc = [torch.empty((cap, H, d), **e) for _ in range(n_in)]          # Qc, Kc, Vc, dOc
         self.idx = torch.empty(max(cap, 1), dtype=torch.int32, device=self.dev)
         self.n_dev = torch.empty(1, dtype=torch.int32, device=self.dev)
+        # N is read by the host once per step.  Where the device can address
+        # pinned host memory, the compaction kernel writes N there and the host
+        # waits on an event: a device-to-host copy of 4 bytes would queue on
+        # the copy engine behind any large transfer already in flight.
+        self.n_host = torch.zeros(1, dtype=torch.int32).pin_memory()
+        self.n_zero_copy = u.device_accessible(self.n_host)
         self.status = torch.zeros(1, dtype=torch.int32, device=self.dev)
         self.ws_compact = torch.empty(max(u.lib().ut_fg_compact_workspace_size(T), 16), dtype=torch.uint8,
                                       device=self.dev)
@@ -53,9 +59,17 @@ class HotPath:
         self.N: Optional[int] = None
 
     def compact(self, mask: torch.Tensor, canvas: list[torch.Tensor]) -> int:
-        u.ut_fg_compact(mask, canvas, capacity=self.T, outs=self.xc[:len(canvas)], idx=self.idx, n_out=self.n_dev,
-                        ws=self.ws_compact, status=self.status)
-        self.N = int(self.n_dev.item())  # the one device-to-host read of a step
+        if self.n_zero_copy:
+            u.ut_fg_compact(mask, canvas, capacity=self.T, outs=self.xc[:len(canvas)], idx=self.idx,
+                            n_out=self.n_host, ws=self.ws_compact, status=self.status)
+            done = torch.cuda.Event()
+            done.record()
+            done.synchronize()
+            self.N = int(self.n_host[0])  # the one device-to-host read of a step
+        else:
+            u.ut_fg_compact(mask, canvas, capacity=self.T, outs=self.xc[:len(canvas)], idx=self.idx,
+                            n_out=self.n_dev, ws=self.ws_compact, status=self.status)
+            self.N = int(self.n_dev.item())  # the one device-to-host read of a step
         return self.N
 
     def views(self, N: int):

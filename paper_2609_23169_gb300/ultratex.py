@@ -25,7 +25,7 @@ EXPORTS = (
     "ut_strerror", "ut_topk_count", "ut_fg_compact_workspace_size", "ut_fg_compact", "ut_fg_scatter",
     "ut_block_mask_workspace_size", "ut_block_mask", "ut_bsattn_fwd", "ut_bsattn_bwd_workspace_size",
     "ut_bsattn_bwd", "ut_fg_compact_noalloc", "ut_fg_euler_update", "ut_fg_composite",
-    "ut_fg_gather_rope", "ut_fg_scatter_rope", "ut_fg_mask_from_alpha",
+    "ut_fg_gather_rope", "ut_fg_scatter_rope", "ut_fg_mask_from_alpha", "ut_device_accessible",
 )
 
 
@@ -98,6 +98,8 @@ def lib() -> ctypes.CDLL:
                                      _i32, _vp]
     L.ut_fg_mask_from_alpha.restype = _i32
     L.ut_fg_mask_from_alpha.argtypes = [_vp, _i32, _i32, _i32, _i32, _i32, _i32, _vp, _vp]
+    L.ut_device_accessible.restype = _i32
+    L.ut_device_accessible.argtypes = [_vp]
     _lib = L
     return L
 
@@ -156,6 +158,12 @@ def attn_shape(x: torch.Tensor, block: int, block_k: int = 0) -> AttnShape:
     return AttnShape(N, H, d, block, _dtype_code(x), x.stride(0), block_k)
 
 
+def device_accessible(t: torch.Tensor) -> bool:
+    """True if the library's kernels can address the tensor's storage directly
+    (device memory, or host memory mapped into the device's address space)."""
+    return bool(lib().ut_device_accessible(_p(t)))
+
+
 def status_word(device=None) -> torch.Tensor:
     return torch.zeros(1, dtype=torch.int32, device=device or "cuda")
 
@@ -190,6 +198,8 @@ def ut_fg_compact(mask: torch.Tensor, srcs: Sequence[torch.Tensor], capacity: Op
         idx = torch.empty(max(cap, 1), dtype=torch.int32, device=dev)
     if n_out is None:
         n_out = torch.empty(1, dtype=torch.int32, device=dev)
+    elif n_out.device.type != "cuda" and not device_accessible(n_out):
+        raise ValueError("n_out must be device memory or host memory the device can address (pinned)")
     L = lib()
     wsb = L.ut_fg_compact_workspace_size(T)
     if ws is None:

@@ -169,6 +169,18 @@ def test_alpha_mask_argument_errors_are_caught_on_host(L):
     assert f(None, 6, 0, 2048, 16, 1, 0, None, None) == u.UT_OK                        # empty image
 
 
+def test_device_accessible_without_device(L):
+    """Null and plain host pointers are never reported as device-accessible;
+    on a machine without a GPU every pointer reads 0 (the query only asks the
+    runtime and never launches)."""
+    import torch
+    from paper_2609_23169_gb300 import ultratex as u
+    assert L.ut_device_accessible(None) == 0
+    assert u.device_accessible(torch.zeros(4, dtype=torch.int32)) is False
+    with pytest.raises(ValueError, match="n_out"):
+        u.ut_fg_compact(torch.ones(4, dtype=torch.uint8), [torch.zeros(4, 4)], n_out=torch.zeros(1, dtype=torch.int32))
+
+
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     from paper_2609_23169_gb300 import ultratex as u
     monkeypatch.setattr(u, "_lib", None)

@@ -65,6 +65,34 @@ def test_compaction_ragged_and_degenerate(T, frac, row):
     assert st == 0 and N == int((mask != 0).sum())
 
 
+def test_device_accessible_query():
+    from paper_2609_23169_gb300 import ultratex as u
+    assert u.device_accessible(torch.zeros(4, device="cuda"))
+    assert u.device_accessible(torch.zeros(4).pin_memory())
+
+
+@pytest.mark.parametrize("T,frac", [(37, 0.5), (70001, 0.3), (5000, 0.0)])
+def test_compaction_count_in_pinned_host_memory(T, frac):
+    """N written straight into pinned host memory matches the device count and
+    the oracle; the gather that reads N back from there copies the same rows."""
+    from paper_2609_23169_gb300 import ultratex as u
+    g = np.random.Generator(np.random.PCG64([5, T]))
+    mask = (g.random(T) < frac).astype(np.uint8)
+    x = torch.from_numpy(g.integers(-2 ** 31, 2 ** 31 - 1, size=(T, 8), dtype=np.int32)).view(torch.float32)
+    m, xd = torch.from_numpy(mask).cuda(), x.cuda()
+    n_host = torch.full((1,), -1, dtype=torch.int32).pin_memory()
+    assert u.device_accessible(n_host)
+    st = u.status_word()
+    idx, _, (out,) = u.ut_fg_compact(m, [xd], n_out=n_host, status=st)
+    done = torch.cuda.Event()
+    done.record()
+    done.synchronize()
+    ref_idx, (ref_rows,) = o.fg_compact(mask, [bits(x)])
+    assert int(n_host[0]) == len(ref_idx) and int(st.item()) == 0
+    assert np.array_equal(idx[:len(ref_idx)].cpu().numpy(), ref_idx)
+    assert np.array_equal(bits(out[:len(ref_idx)]), ref_rows)
+
+
 def test_compaction_capacity_overflow_reports_status():
     from paper_2609_23169_gb300 import ultratex as u
     g = np.random.Generator(np.random.PCG64(9))
