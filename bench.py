@@ -233,9 +233,11 @@ def run_ours(args, rank, world, local_rank):
     # ---- e2e through host buffers: every step copies its canvas inputs from
     # pinned host memory and its canvas results back.  The copies of
     # neighbouring steps overlap the compute of the current one (three sets
-    # of device inputs and outputs); uploads and downloads share one
-    # copy stream, one direction at a time, because the host link moves less
-    # in total when both directions run at once.
+    # of device inputs and outputs).  Whether uploads and downloads should
+    # run at the same time depends on the host link (full duplex on some
+    # hosts, less total bandwidth with both directions at once on others), so
+    # the warm-up times both arrangements -- one copy stream for both
+    # directions, or one per direction -- and the timed steps use the faster.
     e2e = None
     if not args.no_e2e:
         pin_in = [x.pin_memory() for x in (torch.from_numpy(mask_np), q, k, v, do)]
@@ -249,7 +251,10 @@ def run_ours(args, rank, world, local_rank):
         paths = [hp] + [P.HotPath(w.T, w.heads, w.head_dim, w.block, torch.bfloat16, u.UT_MASK_TOPK, rho=w.rho,
                                   device=dev) for _ in range(NB - 1)]
         s_cmp = torch.cuda.Stream(dev)
-        s_up = s_dn = torch.cuda.Stream(dev)   # one copy stream for both directions
+        s_copy = [torch.cuda.Stream(dev), torch.cuda.Stream(dev)]
+        mode = {"split": False}   # False: uploads and downloads share s_copy[0]
+        up_s = lambda: s_copy[0]  # noqa: E731
+        dn_s = lambda: s_copy[1] if mode["split"] else s_copy[0]  # noqa: E731
         ev = lambda: torch.cuda.Event(enable_timing=False)  # noqa: E731
         in_ready = [ev() for _ in range(NB)]
         in_free = [None] * NB
@@ -257,6 +262,7 @@ def run_ours(args, rank, world, local_rank):
 
         def upload(k_):
             b = k_ % NB
+            s_up = up_s()
             with torch.cuda.stream(s_up):
                 if in_free[b] is not None:
                     s_up.wait_event(in_free[b])
@@ -278,6 +284,7 @@ def run_ours(args, rank, world, local_rank):
 
         def download(k_):
             b = k_ % NB
+            s_dn = dn_s()
             with torch.cuda.stream(s_dn):
                 s_dn.wait_event(in_free[b])
                 for hst, dvc in zip(pin_out[b], [paths[b].o_canvas] + paths[b].g_canvas):
@@ -299,21 +306,34 @@ def run_ours(args, rank, world, local_rank):
                     download(k_ - 1)
             download(n_steps - 1)
 
+        def time_e2e(n_steps):
+            torch.cuda.synchronize()
+            s_up, s_dn = up_s(), dn_s()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(s_up)
+            s_cmp.wait_stream(s_up)
+            s_dn.wait_stream(s_up)
+            run(n_steps)
+            s_dn.wait_stream(s_cmp)
+            s_dn.wait_stream(s_up)
+            e1.record(s_dn)
+            torch.cuda.synchronize()
+            return e0.elapsed_time(e1) / n_steps
+
         run(2)
-        torch.cuda.synchronize()
+        trial = {}
+        for split in (False, True):
+            mode["split"] = split
+            trial[split] = time_e2e(max(3, args.warmup))
+        if world > 1:   # every rank takes the arrangement that is faster on the slowest rank
+            t = torch.tensor([trial[False], trial[True]], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            trial = {False: float(t[0]), True: float(t[1])}
+        mode["split"] = trial[True] < trial[False]
         if world > 1:
             dist.barrier()
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(s_up)
-        s_cmp.wait_stream(s_up)
-        s_dn.wait_stream(s_up)
-        run(args.steps)
-        s_dn.wait_stream(s_cmp)
-        s_dn.wait_stream(s_up)
-        e1.record(s_dn)
-        torch.cuda.synchronize()
-        e_ms = e0.elapsed_time(e1) / args.steps
+        e_ms = time_e2e(args.steps)
         for x in paths:
             u.check_status(x.status)
         if world > 1:
@@ -322,8 +342,10 @@ def run_ours(args, rank, world, local_rank):
             e_ms = float(t.item())
         e2e = {"value": round(world * f_step / (e_ms * 1e-3) / 1e12, 3), "unit": "TFLOP/s",
                "ms_per_step": round(e_ms, 3), "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-               "pipeline": "2 streams (copies in both directions, one at a time | compute), 3 sets of device "
-                           "inputs and outputs"}
+               "pipeline": ("3 streams (uploads | downloads | compute)" if mode["split"] else
+                            "2 streams (uploads and downloads, one at a time | compute)") +
+                           ", 3 sets of device inputs and outputs; warm-up ms/step with one copy stream "
+                           f"{trial[False]:.1f}, with one per direction {trial[True]:.1f}"}
 
     peaks, peak_src = load_peaks()
     # DRAM bytes per launch of each entry point from the last ncu capture of the
