@@ -253,3 +253,27 @@ def test_bwd_c1024_sampled():
 
 def test_bwd_c2048_sampled():
     print(_sampled_bwd_check(CONFIGS["c2048"], "topk"))
+
+
+def test_hot_path_count_in_pinned_or_device_memory():
+    """The step reads N either from pinned host memory the device writes (after
+    an event) or by a device-to-host copy; both give the same N and the same
+    canvas results bit for bit."""
+    from paper_2609_23169_gb300 import path as P
+    from paper_2609_23169_gb300 import ultratex as u
+    w = CONFIGS["c512"].with_(heads=2)
+    m = torch.from_numpy(w.canvas_mask()).cuda()
+    q, k, v, do = (x.cuda() for x in (w.q(), w.k(), w.v(), w.dout()))
+    bm = torch.from_numpy(w.block_bitmap()).cuda()
+    outs = []
+    for zero_copy in (True, False):
+        hp = P.HotPath(w.T, w.heads, w.head_dim, w.block, torch.bfloat16, u.UT_MASK_BITMAP, device="cuda")
+        assert hp.n_zero_copy   # pinned host memory is device-accessible on this system
+        hp.n_zero_copy = zero_copy
+        N = hp.step(m, q, k, v, do, bm)
+        torch.cuda.synchronize()
+        u.check_status(hp.status)
+        outs.append((N, [t.view(torch.int16).cpu() for t in [hp.o_canvas] + hp.g_canvas]))
+    assert outs[0][0] == outs[1][0] == w.N
+    for a, b in zip(outs[0][1], outs[1][1]):
+        assert torch.equal(a, b)
