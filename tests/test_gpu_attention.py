@@ -258,7 +258,8 @@ def test_bwd_c2048_sampled():
 def test_hot_path_count_in_pinned_or_device_memory():
     """The step reads N either from pinned host memory the device writes (after
     an event) or by a device-to-host copy; both give the same N and the same
-    canvas results bit for bit."""
+    canvas results: bit for bit for O, dK and dV, and for dQ up to the order
+    of its fp32 reductions."""
     from paper_2609_23169_gb300 import path as P
     from paper_2609_23169_gb300 import ultratex as u
     w = CONFIGS["c512"].with_(heads=2)
@@ -273,7 +274,9 @@ def test_hot_path_count_in_pinned_or_device_memory():
         N = hp.step(m, q, k, v, do, bm)
         torch.cuda.synchronize()
         u.check_status(hp.status)
-        outs.append((N, [t.view(torch.int16).cpu() for t in [hp.o_canvas] + hp.g_canvas]))
+        outs.append((N, [t.cpu() for t in [hp.o_canvas] + hp.g_canvas]))
     assert outs[0][0] == outs[1][0] == w.N
-    for a, b in zip(outs[0][1], outs[1][1]):
-        assert torch.equal(a, b)
+    (o0, dq0, dk0, dv0), (o1, dq1, dk1, dv1) = outs[0][1], outs[1][1]
+    for a, b in ((o0, o1), (dk0, dk1), (dv0, dv1)):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    assert torch.allclose(dq0.float(), dq1.float(), rtol=1e-2, atol=1e-4)
