@@ -108,26 +108,41 @@ __global__ void __launch_bounds__(kSelThreads) score_select_kernel(const float* 
   const float* PK = pooled + (int64_t)H * nq * d + ((int64_t)h * nk) * d;
   for (int t = threadIdx.x; t < rows * d; t += kSelThreads) pq[t] = PQ[(int64_t)i0 * d + t];
   __syncthreads();
-  for (int j = threadIdx.x; j < nk; j += kSelThreads) {
-    float acc[kSelMaxRows];
+  // two key blocks per thread and 16-byte loads of the pooled query rows: one
+  // shared load feeds eight FMAs (the sums are accumulated in the same order
+  // as one column at a time)
+  for (int j0 = threadIdx.x; j0 < nk; j0 += 2 * kSelThreads) {
+    const int j1 = j0 + kSelThreads;
+    const bool has1 = j1 < nk;
+    float acc0[kSelMaxRows], acc1[kSelMaxRows];
 #pragma unroll
-    for (int r = 0; r < kSelMaxRows; ++r) acc[r] = 0.f;
-    const float* kj = PK + (int64_t)j * d;
+    for (int r = 0; r < kSelMaxRows; ++r) acc0[r] = acc1[r] = 0.f;
+    const float* k0 = PK + (int64_t)j0 * d;
+    const float* k1 = PK + (int64_t)(has1 ? j1 : j0) * d;
     for (int e = 0; e < d; e += 4) {
-      float4 kv = *reinterpret_cast<const float4*>(kj + e);
+      const float4 a = *reinterpret_cast<const float4*>(k0 + e);
+      const float4 b = *reinterpret_cast<const float4*>(k1 + e);
 #pragma unroll
       for (int r = 0; r < kSelMaxRows; ++r) {
         if (r < rows) {
-          acc[r] = fmaf(pq[r * d + e + 0], kv.x, acc[r]);
-          acc[r] = fmaf(pq[r * d + e + 1], kv.y, acc[r]);
-          acc[r] = fmaf(pq[r * d + e + 2], kv.z, acc[r]);
-          acc[r] = fmaf(pq[r * d + e + 3], kv.w, acc[r]);
+          const float4 p = *reinterpret_cast<const float4*>(pq + r * d + e);
+          acc0[r] = fmaf(p.x, a.x, acc0[r]);
+          acc0[r] = fmaf(p.y, a.y, acc0[r]);
+          acc0[r] = fmaf(p.z, a.z, acc0[r]);
+          acc0[r] = fmaf(p.w, a.w, acc0[r]);
+          acc1[r] = fmaf(p.x, b.x, acc1[r]);
+          acc1[r] = fmaf(p.y, b.y, acc1[r]);
+          acc1[r] = fmaf(p.z, b.z, acc1[r]);
+          acc1[r] = fmaf(p.w, b.w, acc1[r]);
         }
       }
     }
 #pragma unroll
     for (int r = 0; r < kSelMaxRows; ++r)
-      if (r < rows) sc[r * nk + j] = acc[r];
+      if (r < rows) {
+        sc[r * nk + j0] = acc0[r];
+        if (has1) sc[r * nk + j1] = acc1[r];
+      }
   }
   __syncthreads();
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
