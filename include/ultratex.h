@@ -299,7 +299,8 @@ ut_status ut_bsattn_fwd(const ut_attn_shape* shape, const void* q, const void* k
  *   dq, dk, dv  [N, H, d] outputs (dtype of shape), fully overwritten.
  *   ws          ut_bsattn_bwd_workspace_size(shape) bytes: D and LSE*log2(e)
  *               per head and padded row, and for bf16 an fp32 dQ accumulator
- *               [H, ceil(N/128)*128, d] (about 4*H*N*d bytes).
+ *               [H, ceil(N/128)*128, d] (about 4*H*N*d bytes) followed by
+ *               the counter that hands key blocks to the kernel's CTAs.
  * bf16 runs one fused tensor-core kernel per key block (S and dP computed
  * once per retained pair); dQ is summed over key blocks with fp32 atomic
  * additions, so its last bits may differ between runs (dK, dV do not). */

@@ -78,6 +78,7 @@ struct BwdParams {
   int list_shift;       // 0 (b_q = 128) or 1 (b_q = 64)
   float scale, scale_log2;
   uint64_t timeout_ns;
+  int32_t* item_counter;  // next item to hand out (zeroed before the launch)
 };
 
 // 64 consecutive TMEM columns of this warp's 32 lanes, one wait.
@@ -121,6 +122,14 @@ static_assert(kFuRegCtl + 2 * kFuRegEw + kFuRegDrain == 4 * kFuRegLaunch, "setma
 constexpr int kFuQStages = 2, kFuDoStages = 1;
 constexpr uint32_t kColR0 = 0, kColRQ = 128, kColFuDv = 256, kColFuDk = 384;
 
+// Items are handed out dynamically (the transposed lists differ in length:
+// 36-153 query blocks per key block at the 2048 canvas, so a static
+// round-robin leaves the busiest CTA ~5% above the mean), still in head-major
+// order, so that the CTAs in flight share one head's Q, dO and dQ accumulator
+// in L2.  kItemConsumers: TMA lane 1, the MMA warp, 8 elementwise warps, 4
+// drain warps.
+constexpr int kItemSlots = 4, kItemConsumers = 14;
+
 template <int D>
 struct FusedSmem {
   static constexpr int kC = D / 64;
@@ -138,6 +147,10 @@ struct FusedSmem {
   uint64_t s_full, s_empty, dp_full, dp_empty, pt_full, pt_done, dst_full, ds_done, dq_empty;
   uint64_t acc_full, acc_empty, mma_done;
   uint64_t rowvec_full[2];
+  // the CTA's item sequence: TMA lane 0 takes the next item from the global
+  // counter and publishes it here; every other role reads the slots in order
+  int32_t item[kItemSlots];
+  uint64_t item_full[kItemSlots], item_empty[kItemSlots];
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -191,6 +204,10 @@ __global__ void __launch_bounds__(kFuThreads, 1)
     mbar_init(&sm.mma_done, 1);
     mbar_init(&sm.rowvec_full[0], 256);
     mbar_init(&sm.rowvec_full[1], 256);
+    for (int s = 0; s < kItemSlots; ++s) {
+      mbar_init(&sm.item_full[s], 1);
+      mbar_init(&sm.item_empty[s], kItemConsumers);
+    }
     sm.abort_flag = 0;
     fence_barrier_init();
   }
@@ -202,8 +219,24 @@ __global__ void __launch_bounds__(kFuThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  const int G = gridDim.x;
   const uint32_t wg = warp >> 2;
+  // next item of this CTA's sequence (-1: none left); whole warp (converged)
+  // or, with one = true, a single thread.  Returns false on timeout / abort.
+  auto next_item = [&](uint32_t& kk, int& w, bool one) -> bool {
+    const uint32_t s = kk % kItemSlots, n = kk / kItemSlots;
+    const bool got = one ? mbar_wait(&sm.item_full[s], n & 1, abort_flag, prm.status, prm.timeout_ns)
+                         : warp_wait(&sm.item_full[s], n & 1, abort_flag, prm.status, prm.timeout_ns);
+    if (!got) return false;
+    w = *reinterpret_cast<volatile int32_t*>(&sm.item[s]);
+    if (one) {
+      mbar_arrive(&sm.item_empty[s]);
+    } else {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.item_empty[s]);
+    }
+    ++kk;
+    return true;
+  };
   if (wg == 0) {
     setmaxnreg_dec<kFuRegCtl>();
     if (warp == 0) {
@@ -224,9 +257,22 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         uint8_t* ring = is_q ? &sm.q[0][0] : &sm.dout[0][0];
         const void* tmap = is_q ? static_cast<const void*>(&tm_q) : static_cast<const void*>(&tm_do);
         const uint32_t nst = is_q ? kFuQStages : kFuDoStages;
-        uint32_t ki = 0, qd = 0;
+        uint32_t ki = 0, qd = 0, kk = 0;
         bool ok = true;
-        for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+        for (;;) {
+          int w;
+          if (is_q) {  // take the next item and publish it to the other roles
+            const uint32_t s = kk % kItemSlots, n = kk / kItemSlots;
+            if (!(ok = mbar_wait(&sm.item_empty[s], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+            w = atomicAdd(prm.item_counter, 1);
+            if (w >= prm.n_items) w = -1;
+            *reinterpret_cast<volatile int32_t*>(&sm.item[s]) = w;
+            mbar_arrive(&sm.item_full[s]);
+            ++kk;
+          } else if (!(ok = next_item(kk, w, true))) {
+            break;
+          }
+          if (w < 0) break;
           const int h = w / prm.nq, j = w % prm.nq;
           TileList<kSub> tl;
           tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
@@ -249,6 +295,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
             for (int c = 0; c < C; ++c)
               tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, i * kTile, pol_qd);
           }
+          if (!ok) break;
         }
         auto drain = [&](uint64_t* bar, uint32_t parity) {
           if (!mbar_drain(bar, parity, kDrainTimeoutNs)) set_status(prm.status, UT_ERR_TIMEOUT);
@@ -265,9 +312,11 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         constexpr uint32_t idesc_dq = idesc_bf16_f32(kTile, kTile, true, true);
         const uint32_t k_addr = smem_u32(sm.k), v_addr = smem_u32(sm.v);
       const uint32_t pt_addr = smem_u32(sm.pt), dst_addr = smem_u32(sm.dst);
-        uint32_t ki = 0, qd0 = 0;
+        uint32_t ki = 0, qd0 = 0, kk = 0;
         bool ok = true;
-        for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+        for (;;) {
+          int w;
+          if (!(ok = next_item(kk, w, false)) || w < 0) break;
           TileList<kSub> tl;
           tl.init(prm.ptr, prm.idx, w / prm.nq, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
           const int L = tl.count_warp();
@@ -338,6 +387,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
             mma_commit_w(&sm.ds_done);
             if (t == L - 1) mma_commit_w(&sm.kv_empty);
           }
+          if (!ok) break;
           mma_commit_w(&sm.acc_full);
           qd0 += L;
           ++ki;
@@ -362,10 +412,12 @@ __global__ void __launch_bounds__(kFuThreads, 1)
     const float c = prm.scale_log2;
     const uint32_t pt_row = smem_u32(sm.pt) + half * kChunk + krow * 128;
     const uint32_t dst_row = smem_u32(sm.dst) + half * kChunk + krow * 128;
-    uint32_t qd0 = 0, ki = 0;
+    uint32_t qd0 = 0, ki = 0, kk = 0;
     bool ok = true;
     const uint32_t kh = krow >> 6;  // which 64-row half of the key tile
-    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+    for (;;) {
+      int w;
+      if (!(ok = next_item(kk, w, false)) || w < 0) break;
       const int h = w / prm.nq, j = w % prm.nq;
       TileList<kSub> tl;
       tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
@@ -515,9 +567,11 @@ __global__ void __launch_bounds__(kFuThreads, 1)
     const uint32_t quarter = warp & 3;
     const uint32_t dcol = quarter * 32 + lane;
     const uint32_t lane_base = (quarter * 32) << 16;
-    uint32_t qd0 = 0;
+    uint32_t qd0 = 0, kk = 0;
     bool ok = true;
-    for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
+    for (;;) {
+      int w;
+      if (!(ok = next_item(kk, w, false)) || w < 0) break;
       const int h = w / prm.nq;
       TileList<kSub> tl;
       tl.init(prm.ptr, prm.idx, h, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
@@ -546,6 +600,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
           }
         }
       }
+      if (!ok) break;
       qd0 += L;
     }
   }
@@ -578,7 +633,7 @@ __global__ void __launch_bounds__(256) bwd_dq_finalize_kernel(const float* __res
 // ----------------------------------------------------------------- launcher
 size_t attn_bwd_tc_ws(const AttnProblem& p) {
   const size_t Np = (size_t)((p.N + kTile - 1) / kTile) * kTile;
-  return 2 * (size_t)p.H * Np * sizeof(float) + (size_t)p.H * Np * p.d * sizeof(float);
+  return 2 * (size_t)p.H * Np * sizeof(float) + (size_t)p.H * Np * p.d * sizeof(float) + 16;  // + item counter
 }
 
 constexpr size_t kMaxDynSmem = 232448;  // 227 KB opt-in per block on sm_100/sm_103
@@ -620,7 +675,9 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
   float* lse2 = static_cast<float*>(ws);
   float* dsum = lse2 + (size_t)p.H * Np;
   float* dq_acc = dsum + (size_t)p.H * Np;
-  cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)p.H * Np * p.d * sizeof(float), stream);
+  int32_t* item_counter = reinterpret_cast<int32_t*>(dq_acc + (size_t)p.H * Np * p.d);
+  // one clear for the dQ accumulator and the item counter right after it
+  cudaError_t e = cudaMemsetAsync(dq_acc, 0, (size_t)p.H * Np * p.d * sizeof(float) + 16, stream);
   if (e != cudaSuccess) return e;
   bwd_pre_kernel<<<(unsigned)((Np + 7) / 8), 256, 0, stream>>>(
       static_cast<const __nv_bfloat16*>(o), static_cast<const __nv_bfloat16*>(dout), lse, p.N, Np, p.H, p.d,
@@ -652,6 +709,7 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
   a.scale = p.scale;
   a.scale_log2 = p.scale * 1.4426950408889634f;
   a.timeout_ns = timeout_ns;
+  a.item_counter = item_counter;
   __nv_bfloat16* dqb = static_cast<__nv_bfloat16*>(dq);
   const bool sub = p.block == 64 || p.block_k == 64;
   if (p.d == 64)
