@@ -351,9 +351,9 @@ def run_ours(args, rank, world, local_rank):
     # DRAM bytes per launch of each entry point from the last ncu capture of the
     # current kernels (summarised under profiles/), taken at 8 heads and scaled
     # to 24 (each head is an independent problem of the same size); only valid
-    # for the 24-head 2048 workload.  Backward: fused kernel 14.44 GB + dQ
+    # for the 24-head 2048 workload.  Backward: fused kernel 6.08 GB + dQ
     # finalize 0.49 GB + D/LSE pre-pass 0.36 GB + accumulator clear 0.35 GB.
-    traffic_24h = {"bsattn_fwd": 2.60e9, "bsattn_bwd": 46.9e9}
+    traffic_24h = {"bsattn_fwd": 2.60e9, "bsattn_bwd": 21.8e9}
     # dominant kernel by measured time
     dom = max(("bsattn_fwd", "bsattn_bwd"), key=lambda n: kern_ms.get(n, 0))
     dom_flops = f_fwd if dom == "bsattn_fwd" else 2.5 * f_fwd
