@@ -107,6 +107,24 @@ def test_argument_errors_are_caught_on_host(L):
                            bogus, bogus, bogus, bogus, 1 << 20, None, None) == u.UT_ERR_INVALID_ARG
 
 
+def test_backward_workspace_holds_accumulator_and_counter(L):
+    """The bf16 backward's workspace covers D and LSE*log2e per padded row, the
+    fp32 dQ accumulator and the key-block counter after it; one byte less is
+    refused before any launch (the pointers are also misaligned, a second
+    reason to refuse)."""
+    from paper_2609_23169_gb300 import ultratex as u
+    S = ctypes.byref
+    N, H, d = 1000, 2, 128
+    sh = _shape(u, N=N, H=H, d=d, b=128, dtype=u.UT_BF16)
+    Np = -(-N // 128) * 128
+    need = 2 * H * Np * 4 + H * Np * d * 4 + 16
+    wsb = L.ut_bsattn_bwd_workspace_size(S(sh))
+    assert wsb >= need
+    bad = ctypes.c_void_p(16 * 1024 + 8)
+    assert L.ut_bsattn_bwd(S(sh), bad, bad, bad, bad, bad, bad, bad, bad, bad, bad, 0.1, bad, bad, bad,
+                           ctypes.c_void_p(16 * 1024), need - 1, None, None) == u.UT_ERR_INVALID_ARG
+
+
 def test_sampler_argument_errors_are_caught_on_host(L):
     from paper_2609_23169_gb300 import ultratex as u
     bogus = ctypes.c_void_p(16 * 1024)   # never dereferenced: every call must fail validation first
