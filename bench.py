@@ -12,8 +12,13 @@ e2e    = the same FLOPs / time of the step through the public API with the
          canvas inputs in pinned host memory: host->device copies of the
          mask and Q, K, V, dO, the step, and device->host copies of O, dQ,
          dK, dV canvases inside the timed region.
-The reference arm (--impl reference) times the fp64 CPU oracle on a bounded
-sample of the same workload (this build has no reference implementation).
+per_config  the same step on the 512 and 1024 canvases (structured block
+         lists), L2 flushed before each step.
+The reference arm (--impl reference) and cpu_baseline time the fp64 CPU
+oracle on a bounded sample of the same workload, counting the same work per
+retained pair as the GPU value (forward + full backward, 14*d FLOP per
+query-key row pair); oracle_times records the oracle's wall time on whole
+configurations (this build has no reference implementation).
 """
 from __future__ import annotations
 
@@ -53,6 +58,10 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-per-config", action="store_true", help="skip the 512 / 1024 canvas steps")
+    ap.add_argument("--no-oracle-times", action="store_true", help="skip the whole-config oracle wall times")
+    ap.add_argument("--oracle-time", default="", help=argparse.SUPPRESS)  # internal: one oracle timing run
+    ap.add_argument("--oracle-parts", default="fwd,bwd", help=argparse.SUPPRESS)
     ap.add_argument("--sweep", action="store_true",
                     help="2048-canvas sweep: one JSON line per (foreground, rho, block) point instead of the bench line")
     return ap.parse_args()
@@ -150,6 +159,181 @@ def whole_job(ms_local: float, flops_local: float, world: int, device=None):
     return float(t.item()), float(f.item())
 
 
+METRIC = "retained-block attention TFLOP/s and % of GB300 bf16 peak at 2048 canvas (~213K tokens)"
+
+
+def workload_config(w, N: int, density: float, world: int) -> dict:
+    """config object of the JSON line; both arms build it from here so that
+    the same workload gives the same object."""
+    rule = (f"Top-K rho={w.rho}" if w.mask_mode == "topk" else "structured lists (own view, partner view, reference)")
+    return {"workload": f"{w.name}: {w.n_images} images x {w.side}x{w.side} tokens (T={w.T}), "
+                        f"{int(round(w.fg_frac * 100))}% {w.shape} foreground (N={N}), H={w.heads}, d={w.head_dim}, "
+                        f"b={w.block}, {rule} (density {density:.4f}), forward+backward",
+            "N": N, "T": w.T, "heads": w.heads, "head_dim": w.head_dim, "block": w.block,
+            "rho": w.rho if w.mask_mode == "topk" else None, "parallelism": f"replicas x{world}",
+            "l2": l2_note(w)}
+
+
+def l2_note(w) -> str:
+    gb = w.T * w.heads * w.head_dim * 2 / 1e9
+    if gb > 0.129:
+        return "inputs larger than L2 (each canvas tensor %.2f GB > 129 MB)" % gb
+    return "L2 flushed before each step by a 256 MB write (each canvas tensor %.3f GB < 129 MB)" % gb
+
+
+def list_density(w, N: int) -> float:
+    """Retained fraction of the block pairs; for Top-K it is K_rho / N_k in every head."""
+    nq = -(-N // w.block)
+    if w.mask_mode == "topk":
+        return max(1, int(math.floor(w.rho * nq))) / nq
+    return float(w.block_bitmap().mean())
+
+
+class StepRunner:
+    """One HotPath on one workload with resident inputs; times whole steps and
+    the entry points inside them with CUDA events on the launching stream."""
+
+    def __init__(self, w, dev):
+        import torch
+        from paper_2609_23169_gb300 import path as P
+        from paper_2609_23169_gb300 import ultratex as u
+        self.w, self.dev, self.u = w, dev, u
+        self.mask_np, q, k, v, do = make_inputs(w, dev)
+        self.host = (q, k, v, do)
+        self.mask = torch.from_numpy(self.mask_np).to(dev)
+        self.tq, self.tk, self.tv, self.tdo = (x.to(dev) for x in (q, k, v, do))
+        topk = w.mask_mode == "topk"
+        self.mode = u.UT_MASK_TOPK if topk else u.UT_MASK_BITMAP
+        self.bitmap = None if topk else torch.from_numpy(w.block_bitmap()).to(dev)
+        self.hp = P.HotPath(w.T, w.heads, w.head_dim, w.block, torch.bfloat16, self.mode,
+                            rho=w.rho if topk else 0.0, device=dev)
+        self.stream = torch.cuda.current_stream()
+        self.ev = {}
+
+    def timed(self, name, fn):
+        import torch
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(self.stream)
+        r = fn()
+        b.record(self.stream)
+        self.ev.setdefault(name, []).append((a, b))
+        return r
+
+    def step(self, record: bool) -> int:
+        hp = self.hp
+        inputs = [self.tq, self.tk, self.tv, self.tdo]
+        if not record:
+            return hp.step(self.mask, *inputs, bitmap=self.bitmap)
+        N = self.timed("compact", lambda: hp.compact(self.mask, inputs))
+        self.timed("block_mask", lambda: hp.block_lists(N, self.bitmap))
+        self.timed("bsattn_fwd", lambda: hp.forward(N))
+        self.timed("bsattn_bwd", lambda: hp.backward_pass(N))
+        self.timed("scatter", lambda: hp.scatter(N))
+        return N
+
+    def lists_flops(self, N: int):
+        w, hp = self.w, self.hp
+        nq = -(-N // w.block)
+        rp = hp.row_ptr[:w.heads * nq + 1].cpu().numpy()
+        ci = hp.col_idx[:int(rp[-1])].cpu().numpy()
+        f_fwd = retained_flops(rp, ci, N, w.block, w.head_dim)
+        density = float(rp[-1]) / (w.heads * nq * nq)
+        return f_fwd, density
+
+    def kernel_ms(self) -> dict:
+        return {n: sum(a.elapsed_time(b) for a, b in l) / len(l) for n, l in self.ev.items()}
+
+
+def time_per_config(names, dev, steps: int, warmup: int, peak: float) -> dict:
+    """The whole step on the smaller canvases (structured block lists), timed
+    step by step with the L2 flushed (a 256 MB write) before each step: the
+    512 canvas's tensors are smaller than L2."""
+    import torch
+    from synth import CONFIGS
+    out = {}
+    flush = torch.empty(64 << 20, dtype=torch.float32, device=dev)
+    for name in names:
+        w = CONFIGS[name]
+        r = StepRunner(w, dev)
+        for _ in range(warmup):
+            N = r.step(False)
+        torch.cuda.synchronize()
+        r.u.check_status(r.hp.status)
+        f_fwd, density = r.lists_flops(N)
+        tot = 0.0
+        for _ in range(steps):
+            flush.fill_(1.0)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(r.stream)
+            r.step(True)
+            e1.record(r.stream)
+            torch.cuda.synchronize()
+            tot += e0.elapsed_time(e1)
+        r.u.check_status(r.hp.status)
+        ms = tot / steps
+        km = r.kernel_ms()
+        tf = 3.5 * f_fwd / (ms * 1e-3) / 1e12
+        out[name] = {"workload": workload_config(w, N, density, 1)["workload"], "N": N,
+                     "ms_per_step": round(ms, 4), "tflops": round(tf, 2), "pct_of_burst_peak": round(100 * tf / peak, 2),
+                     "retained_fwd_tflop": round(f_fwd / 1e12, 4),
+                     "bsattn_fwd": {"ms": round(km["bsattn_fwd"], 4),
+                                    "tflops": round(f_fwd / (km["bsattn_fwd"] * 1e-3) / 1e12, 2)},
+                     "bsattn_bwd": {"ms": round(km["bsattn_bwd"], 4),
+                                    "tflops": round(2.5 * f_fwd / (km["bsattn_bwd"] * 1e-3) / 1e12, 2)},
+                     "l2": "flushed before each step (256 MB write)", "steps": steps}
+        del r
+        torch.cuda.empty_cache()
+    return out
+
+
+def load_traffic_record():
+    """DRAM bytes per launch of the attention entry points from the committed
+    ncu summary (profiles/dram_traffic.txt): one line per entry point with the
+    workload and head count it was captured on, the bytes, and the SHA-256 of
+    the kernel sources at capture time."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    rec = {}
+    if not os.path.exists(path):
+        return rec
+    with open(path) as f:
+        for line in f:
+            parts = line.split()
+            if len(parts) >= 5 and parts[0] in ("bsattn_fwd", "bsattn_bwd") and not line.startswith("#"):
+                rec[parts[0]] = {"workload": parts[1], "heads": int(parts[2]), "bytes": float(parts[3]),
+                                 "sha256": parts[4]}
+    return rec
+
+
+KERNEL_SOURCES = {"bsattn_fwd": ["attn_fwd_tc.cu", "common.cuh"],
+                  "bsattn_bwd": ["attn_bwd_tc.cu", "common.cuh"]}
+
+
+def kernel_source_hash(entry: str) -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES[entry]:
+        with open(os.path.join(ROOT, "paper_2609_23169_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_for(entry: str, w) -> tuple:
+    """(bytes per launch or None, note).  The recorded capture is scaled by the
+    head count (each head is an independent problem of the same size); it is
+    withheld when the kernel sources changed since the capture or the
+    workload differs."""
+    rec = load_traffic_record().get(entry)
+    if rec is None:
+        return None, "no ncu record"
+    if rec["sha256"] != kernel_source_hash(entry):
+        return None, "kernel sources changed since the ncu capture"
+    if rec["workload"] != w.name:
+        return None, f"ncu capture is of {rec['workload']}, not {w.name}"
+    return rec["bytes"] * w.heads / rec["heads"], f"ncu, {rec['heads']}-head capture scaled to {w.heads} heads"
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -168,50 +352,22 @@ def run_ours(args, rank, world, local_rank):
     w = CONFIGS[args.workload]
     if args.heads:
         w = w.with_(heads=args.heads)
-    assert w.mask_mode == "topk", "the benchmark workload uses the Top-K rule"
-    mask_np, q, k, v, do = make_inputs(w, dev)
-    mask = torch.from_numpy(mask_np).to(dev)
-    tq, tk, tv, tdo = (x.to(dev) for x in (q, k, v, do))
-    hp = P.HotPath(w.T, w.heads, w.head_dim, w.block, torch.bfloat16, u.UT_MASK_TOPK, rho=w.rho, device=dev)
-    stream = torch.cuda.current_stream()
-
-    ev = {}
-
-    def timed(name, fn):
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        r = fn()
-        b.record(stream)
-        ev.setdefault(name, []).append((a, b))
-        return r
-
-    def step(record):
-        if not record:
-            return hp.step(mask, tq, tk, tv, tdo)
-        N = timed("compact", lambda: hp.compact(mask, [tq, tk, tv, tdo]))
-        timed("block_mask", lambda: hp.block_lists(N))
-        timed("bsattn_fwd", lambda: hp.forward(N))
-        timed("bsattn_bwd", lambda: hp.backward_pass(N))
-        timed("scatter", lambda: hp.scatter(N))
-        return N
+    r = StepRunner(w, dev)
+    hp, stream, mask_np, mask = r.hp, r.stream, r.mask_np, r.mask
+    q, k, v, do = r.host
+    tq, tk, tv, tdo = r.tq, r.tk, r.tv, r.tdo
 
     for _ in range(args.warmup):
-        N = step(False)
+        N = r.step(False)
     torch.cuda.synchronize()
     u.check_status(hp.status)
-    rp = hp.row_ptr[:w.heads * hp.nq_cap + 1].cpu().numpy()
-    nq = -(-N // w.block)
-    rp = rp[:w.heads * nq + 1]
-    ci = hp.col_idx[:int(rp[-1])].cpu().numpy()
-    f_fwd = retained_flops(rp, ci, N, w.block, w.head_dim)
+    f_fwd, density = r.lists_flops(N)
     f_step = 3.5 * f_fwd
-    density = float(rp[-1]) / (w.heads * nq * nq)
 
     clocks = ClockSampler(local_rank)
     clocks.start()
     time.sleep(0.3)
-    ev.clear()
+    r.ev.clear()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -219,7 +375,7 @@ def run_ours(args, rank, world, local_rank):
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record(stream)
     for _ in range(args.steps):
-        step(True)
+        r.step(True)
     t1.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -227,7 +383,7 @@ def run_ours(args, rank, world, local_rank):
     ms_total = t0.elapsed_time(t1)
     clk = clocks.stop()
     u.check_status(hp.status)
-    kern_ms = {n: sum(a.elapsed_time(b) for a, b in l) / len(l) for n, l in ev.items()}
+    kern_ms = r.kernel_ms()
 
     # whole-job: max time over ranks, FLOPs summed over ranks (replicas)
     ms_total, flops_total = whole_job(ms_total, f_step * args.steps, world, dev)
@@ -252,8 +408,8 @@ def run_ours(args, rank, world, local_rank):
         d2h = sum(x.numel() * x.element_size() for x in pin_out[0])
         dev_in = [[mask, tq, tk, tv, tdo]] + [[torch.empty_like(x) for x in (mask, tq, tk, tv, tdo)]
                                               for _ in range(NB - 1)]
-        paths = [hp] + [P.HotPath(w.T, w.heads, w.head_dim, w.block, torch.bfloat16, u.UT_MASK_TOPK, rho=w.rho,
-                                  device=dev) for _ in range(NB - 1)]
+        paths = [hp] + [P.HotPath(w.T, w.heads, w.head_dim, w.block, torch.bfloat16, r.mode,
+                                  rho=w.rho if w.mask_mode == "topk" else 0.0, device=dev) for _ in range(NB - 1)]
         s_cmp = torch.cuda.Stream(dev)
         s_copy = [torch.cuda.Stream(dev), torch.cuda.Stream(dev)]
         mode = {"split": False}   # False: uploads and downloads share s_copy[0]
@@ -281,7 +437,7 @@ def run_ours(args, rank, world, local_rank):
                 if out_free[b] is not None:
                     s_cmp.wait_event(out_free[b])
                 m_, q_, k2, v_, d_ = dev_in[b]
-                paths[b].step(m_, q_, k2, v_, d_)
+                paths[b].step(m_, q_, k2, v_, d_, bitmap=r.bitmap)
                 done = ev()
                 done.record(s_cmp)
                 in_free[b] = done
@@ -352,34 +508,43 @@ def run_ours(args, rank, world, local_rank):
                            f"{trial[False]:.1f}, with one per direction {trial[True]:.1f}"}
 
     peaks, peak_src = load_peaks()
-    # DRAM bytes per launch of each entry point from the last ncu capture of the
-    # current kernels (summarised under profiles/), taken at 8 heads and scaled
-    # to 24 (each head is an independent problem of the same size); only valid
-    # for the 24-head 2048 workload.  Backward: fused kernel 6.08 GB + dQ
-    # finalize 0.49 GB + D/LSE pre-pass 0.36 GB + accumulator clear 0.35 GB.
-    traffic_24h = {"bsattn_fwd": 2.60e9, "bsattn_bwd": 21.8e9}
-    # dominant kernel by measured time
+    # dominant entry point by measured time
     dom = max(("bsattn_fwd", "bsattn_bwd"), key=lambda n: kern_ms.get(n, 0))
     dom_flops = f_fwd if dom == "bsattn_fwd" else 2.5 * f_fwd
     achieved = dom_flops / (kern_ms[dom] * 1e-3) / 1e12
+    # the step runs for seconds under the power cap, so the dominant kernel is
+    # held against the sustained peak; the burst fraction is reported beside it
     peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    burst = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    traffic, traffic_note = traffic_for(dom, w)
+    # algorithmic bytes of the dominant entry point: forward reads Q, K, V once
+    # and writes O, LSE; backward reads Q, K, V, O, dO, LSE and writes dQ, dK, dV
+    row = N * w.heads * w.head_dim * 2
+    alg_bytes = (4 * row + 4 * w.heads * N) if dom == "bsattn_fwd" else (8 * row + 4 * w.heads * N)
     bytes_tensor = 2 * N * w.heads * w.head_dim * 2 + w.T + 4 * N   # per tensor, compaction
     kernels = {
         n: {"ms": round(kern_ms[n], 4)} for n in kern_ms
     }
     kernels["bsattn_fwd"]["tflops"] = round(f_fwd / (kern_ms["bsattn_fwd"] * 1e-3) / 1e12, 2)
     kernels["bsattn_bwd"]["tflops"] = round(2.5 * f_fwd / (kern_ms["bsattn_bwd"] * 1e-3) / 1e12, 2)
+    for n in ("bsattn_fwd", "bsattn_bwd"):
+        kernels[n]["frac_burst"] = round(kernels[n]["tflops"] / burst, 4)
     kernels["compact"]["gbs"] = round(4 * bytes_tensor / (kern_ms["compact"] * 1e-3) / 1e9, 1)
     sc_bytes = 2 * N * w.heads * w.head_dim * 2 + 3 * (2 * N * w.heads * w.head_dim * 2 +
                                                       (w.T - N) * w.heads * w.head_dim * 2)
     kernels["scatter"]["gbs"] = round(sc_bytes / (kern_ms["scatter"] * 1e-3) / 1e9, 1)
 
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    for n, b_ in (("compact", 4 * bytes_tensor), ("scatter", sc_bytes)):
+        kernels[n]["frac_hbm"] = round(kernels[n]["gbs"] / hbm_peak, 4)
+    per_config = None
+    if rank == 0 and not args.no_per_config and w.name == "c2048" and not args.heads:
+        per_config = time_per_config(("c512", "c1024"), dev, max(3, min(args.steps, 10)), 3, burst)
     sampler = time_sampler_steps(w, dev, hbm_peak) if rank == 0 else None
     rope = time_rope(w, dev, hbm_peak) if rank == 0 else None
     alpha_mask = time_mask_from_alpha(w, dev, hbm_peak) if rank == 0 else None
     line = {
-        "metric": "retained-block attention TFLOP/s and % of GB300 bf16 peak at 2048 canvas (~213K tokens)",
+        "metric": METRIC,
         "value": round(value, 3),
         "unit": "TFLOP/s",
         "n_gpus": world,
@@ -391,22 +556,21 @@ def run_ours(args, rank, world, local_rank):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic",
-        "config": {"workload": f"{w.name}: 13 images x {w.side}x{w.side} tokens (T={w.T}), "
-                               f"{int(w.fg_frac*100)}% blob foreground (N={N}), H={w.heads}, d={w.head_dim}, "
-                               f"b={w.block}, Top-K rho={w.rho} (density {density:.4f}), forward+backward",
-                   "N": N, "T": w.T, "heads": w.heads, "head_dim": w.head_dim, "block": w.block, "rho": w.rho,
-                   "retained_fwd_tflop": round(f_fwd / 1e12, 4), "parallelism": f"replicas x{world}",
-                   "l2": "inputs larger than L2 (each canvas tensor 1.31 GB > 129 MB)"},
+        "config": workload_config(w, N, density, world),
+        "retained_fwd_tflop": round(f_fwd / 1e12, 4),
         "pct_of_peak": round(100 * value / world / peak, 2),
+        "pct_of_burst_peak": round(100 * value / world / burst, 2),
         "roofline": {"bound": "tensor", "kernel": dom, "achieved": round(achieved, 2), "peak": peak,
-                     "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
-                     "traffic": traffic_24h.get(dom) if (w.heads == 24 and w.name == "c2048") else None,
-                     "peak_source": f"{peak_src} bf16 sustained"},
+                     "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "frac_burst": round(achieved / burst, 4),
+                     "traffic": traffic, "traffic_note": traffic_note, "algorithmic_bytes": int(alg_bytes),
+                     "peak_source": f"{peak_src} bf16 sustained (burst {burst})"},
         "kernels": kernels,
         "e2e": e2e,
         "gpu_launches": args.steps * hp_launches(hp),
         "clocks": clk,
     }
+    if per_config is not None:
+        line["per_config"] = per_config
     if sampler is not None:
         line["sampler_steps"] = sampler
     if rope is not None:
@@ -539,37 +703,114 @@ def hp_launches(hp) -> int:
 
 
 # ------------------------------------------------------------------- oracle
-def oracle_sample(w, seconds: float):
-    """Time the fp64 oracle on a bounded sample: whole query blocks of head 0,
-    forward and dQ rows, until `seconds` have passed.  Returns (TFLOP/s, desc)."""
+def oracle_inputs(w, head: int = 0):
+    """Compacted inputs of one head (fp64, the exact bf16 values) and that
+    head's block lists: the oracle's own Top-K lists, or the bitmap's CSR."""
     import torch
     import oracle.ultratex_oracle as o
-    mask = w.canvas_mask()
-    idx = np.flatnonzero(mask)
+    idx = np.flatnonzero(w.canvas_mask())
     t = torch.from_numpy(idx)
-    h = 0
-    qc, kc, vc, dc = (x[t][:, h:h + 1].float().numpy().astype(np.float64) for x in (w.q(), w.k(), w.v(), w.dout()))
+    xs = [x[t][:, head:head + 1].float().numpy().astype(np.float64) for x in (w.q(), w.k(), w.v(), w.dout())]
     N = len(idx)
+    if w.mask_mode == "topk":
+        rp, ci, _, _ = o.topk_block_mask(xs[0], xs[1], w.block, w.rho)
+    else:
+        rp, ci = o.bitmap_to_csr(w.block_bitmap()[head:head + 1])
+    return xs, np.asarray(rp, np.int64), np.asarray(ci, np.int64), N
+
+
+def oracle_sample(w, seconds: float, prepared=None):
+    """Time the fp64 oracle, as it stands, on a bounded sample of the workload:
+    the forward and the full backward (dQ, dK, dV) of a seeded set of whole
+    query blocks of head 0 over their own key-block lists, sized to take about
+    `seconds`.  The work is counted as the GPU value counts it: 14*d FLOP per
+    retained query-key row pair (forward 4*d, backward 2.5x).  Returns
+    (TFLOP/s, description, seconds)."""
+    import oracle.ultratex_oracle as o
+    (qc, kc, vc, dc), rp, ci, N = prepared if prepared is not None else oracle_inputs(w)
     b = w.block
-    rp, ci, _, kr = o.topk_block_mask(qc, kc, b, w.rho)
     nq = -(-N // b)
-    t0 = time.perf_counter()
-    flops = 0.0
-    done = 0
-    for i in range(nq):
-        rows = np.arange(i * b, min(N, (i + 1) * b))
-        o.bsattn_fwd_rows(qc, kc, vc, rp, ci, b, 0, rows)
-        o.bsattn_bwd_dq_rows(qc, kc, vc, dc, rp, ci, b, 0, rows)
-        keys = sum(min(b, N - j * b) for j in ci[rp[i]:rp[i + 1]])
-        # forward (4 d per pair) + dQ part of the backward (dP, dS, dQ: 4 d per pair)
-        flops += 8.0 * w.head_dim * len(rows) * keys
-        done += 1
-        if time.perf_counter() - t0 > seconds:
-            break
-    dt = time.perf_counter() - t0
-    desc = (f"fp64 numpy oracle, head 0, {done} of {nq} query blocks (x{len(rows)} rows) of {w.name}: "
-            f"forward + dQ rows against their {kr} Top-K key blocks; mask/pool/Top-K excluded")
+    sizes = np.array([len(o.tile_rows(j, N, b)) for j in range(nq)], dtype=np.float64)
+    order = np.random.Generator(np.random.PCG64([w.seed, 6])).permutation(nq)
+
+    def run(blocks):
+        keep = np.zeros(nq, dtype=bool)
+        keep[blocks] = True
+        lens = np.where(keep, np.diff(rp), 0)
+        rps = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+        cis = np.concatenate([ci[rp[i]:rp[i + 1]] for i in sorted(blocks)]).astype(np.int64)
+        t0 = time.perf_counter()
+        o.bsattn_fwd(qc, kc, vc, rps, cis, b)
+        o.bsattn_bwd(qc, kc, vc, dc, rps, cis, b)
+        dt = time.perf_counter() - t0
+        pairs = sum(sizes[i] * sizes[ci[rp[i]:rp[i + 1]]].sum() for i in blocks)
+        return dt, 14.0 * w.head_dim * pairs
+
+    dt1, _ = run(order[:1])
+    m = int(max(1, min(nq, seconds / max(dt1, 1e-3))))
+    dt, flops = run(order[:m])
+    kr = int(np.diff(rp).max()) if len(rp) > 1 else 0
+    desc = (f"fp64 numpy oracle (bsattn_fwd + bsattn_bwd as they stand), head 0, {m} seeded query blocks of "
+            f"{nq} of {w.name} with their lists (up to {kr} key blocks each); 14*d FLOP per retained row pair, "
+            f"as the GPU value counts; lists built beforehand, not timed")
     return flops / dt / 1e12, desc, dt
+
+
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.machine()
+
+
+def oracle_time_config(name: str, parts: str) -> dict:
+    """Wall time of the oracle on a whole configuration (all heads): the
+    forward, then the backward (which recomputes its softmax rows).  Lists
+    come from the bitmap (structured configs); compacted inputs in fp64."""
+    import torch
+    import oracle.ultratex_oracle as o
+    from synth import CONFIGS
+    w = CONFIGS[name]
+    idx = np.flatnonzero(w.canvas_mask())
+    t = torch.from_numpy(idx)
+    qc, kc, vc, dc = (x[t].double().numpy() for x in (w.q(), w.k(), w.v(), w.dout()))
+    rp, ci = o.bitmap_to_csr(w.block_bitmap())
+    out = {"N": len(idx), "heads": w.heads}
+    if "fwd" in parts:
+        t0 = time.perf_counter()
+        o.bsattn_fwd(qc, kc, vc, rp, ci, w.block)
+        out["fwd_s"] = round(time.perf_counter() - t0, 3)
+    if "bwd" in parts:
+        t0 = time.perf_counter()
+        o.bsattn_bwd(qc, kc, vc, dc, rp, ci, w.block)
+        out["bwd_s"] = round(time.perf_counter() - t0, 3)
+    return out
+
+
+def oracle_wall_times(cores: int) -> dict:
+    """The oracle's wall time on the tiny, 512 and 1024 configurations in full
+    with every host core, and on tiny and 512 with one thread, each in a fresh
+    interpreter whose BLAS / OpenMP thread count is set before numpy loads."""
+    runs = [("tiny", cores), ("c512", cores), ("c1024", cores), ("tiny", 1), ("c512", 1)]
+    out = {"cores": cores, "cpu_model": cpu_model(), "note": "fp64 numpy oracle, forward then full backward"}
+    for name, threads in runs:
+        env = dict(os.environ)
+        for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
+            env[var] = str(threads)
+        cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--oracle-time", name]
+        try:
+            r = subprocess.run(cmd, capture_output=True, text=True, env=env, timeout=900)
+            rec = json.loads(r.stdout.strip().splitlines()[-1])
+        except Exception as e:  # noqa: BLE001  (a timing that failed is reported as such)
+            rec = {"error": str(e)[:200]}
+        rec["threads"] = threads
+        out[f"{name}_{threads}t"] = rec
+    return out
 
 
 def run_sweep(args):
@@ -652,23 +893,30 @@ def main():
     from synth import CONFIGS
     if args.sweep:
         return run_sweep(args)
+    if args.oracle_time:
+        print(json.dumps(oracle_time_config(args.oracle_time, args.oracle_parts)))
+        return 0
     if args.impl == "reference":
         if rank != 0:
             return 0
         w = CONFIGS[args.workload]
-        per = max(2.0, 60.0 / max(1, args.steps + args.warmup))
-        vals = []
+        prepared = oracle_inputs(w)
+        N = prepared[3]
+        per = max(2.0, min(10.0, 100.0 / max(1, args.steps + args.warmup)))
+        vals, secs = [], []
         for s in range(args.warmup + args.steps):
-            v, desc, dt = oracle_sample(w, per)
+            v, desc, dt = oracle_sample(w, per, prepared)
             if s >= args.warmup:
                 vals.append(v)
+                secs.append(dt)
         val = float(np.mean(vals))
-        line = {"impl": "reference", "metric": "retained-block attention TFLOP/s and % of GB300 bf16 peak at 2048 canvas (~213K tokens)",
+        line = {"impl": "reference", "metric": METRIC,
                 "value": round(val, 6), "unit": "TFLOP/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-                "config": {"workload": w.name}, "ms_per_step": None,
+                "config": workload_config(w, N, list_density(w, N), 1),
+                "ms_per_step": round(1e3 * float(np.mean(secs)), 1),
                 "cpu_baseline": {"value": round(val, 6), "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
-                                 "sample": desc},
+                                 "sample": desc + f"; one sample per step, ~{per:.0f} s each"},
                 "e2e": {"value": round(val, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
         print(json.dumps(line))
         return 0
@@ -681,6 +929,8 @@ def main():
             v, desc, dt = oracle_sample(w, args.cpu_seconds)
             line["cpu_baseline"] = {"value": round(v, 6), "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
                                     "sample": desc + f" ({dt:.1f} s)"}
+        if not args.no_oracle_times and world == 1:
+            line["oracle_times"] = oracle_wall_times(cpu_cores())
         print(json.dumps(line))
     if world > 1:
         import torch.distributed as dist

@@ -120,14 +120,19 @@ ut_status ut_fg_compact(const uint8_t* mask, int64_t T, int32_t n_tensors,
  * this entry point exists for callers that cannot allocate device memory
  * (a host that owns every allocation and passes the library only its inputs
  * and outputs, or a loop that must not enter an allocator).  Same arguments
- * and results as ut_fg_compact, minus ws / ws_bytes.  Its scratch is a fixed
- * 4 KiB device array inside the library (held by every GPU that loads it
- * until exit), so T is limited to 4,194,304 canvas tokens; a larger T
- * returns UT_ERR_UNSUPPORTED before anything is enqueued.  The first call on
- * a device looks up the array's address with that device current; make it
- * before any stream capture.  All calls share the array: calls that overlap
- * on the GPU race and must be serialised by the caller.  No allocation,
- * free or allocating library routine is called. */
+ * and results as ut_fg_compact, minus ws / ws_bytes (T = 0 writes N = 0;
+ * N > capacity reports UT_ERR_CAPACITY in dev_status as there).  Its scratch
+ * is a fixed 4 KiB device array inside the library (held by every GPU that
+ * loads it until exit), so T is limited to 4,194,304 canvas tokens; a larger
+ * T returns UT_ERR_UNSUPPORTED before anything is enqueued.  The first call
+ * in each CUDA context looks up the array's address in that context (cached
+ * under the context's unique id, so a context created later, e.g. after
+ * cudaDeviceReset, gets its own lookup); that first call may also make the
+ * CUDA runtime load the library's device code into the context, which
+ * allocates inside the driver.  Make it before any stream capture.  All calls
+ * in a context share the array: calls that overlap on the GPU race and must
+ * be serialised by the caller.  The entry point itself calls no allocation,
+ * free or allocating library routine. */
 ut_status ut_fg_compact_noalloc(const uint8_t* mask, int64_t T, int32_t n_tensors,
                                 const void* const* h_src, void* const* h_dst, int64_t row_bytes,
                                 int64_t capacity, int32_t* idx_out, int32_t* n_out,

@@ -10,13 +10,20 @@
 // library instead, so the call needs nothing beyond its inputs and outputs.
 //
 // The array is a file-scope __device__ variable: every GPU that loads the
-// library holds it (4 KiB) until the process exits.  Its device address is
-// looked up once per device, on that device's first call, with the device
-// current; make that first call before any stream capture.  All calls on a
-// device share the one array, so calls that overlap on the GPU (different
-// streams, or different host threads without ordering) race on it; serialise
-// them.  The counts are fully rewritten by every call (nothing in the array
-// has to start at zero).
+// library holds it (4 KiB) until the process exits.  In host code its name
+// is only a host-side stand-in, so its device address is looked up with
+// cudaGetSymbolAddress once per CUDA context, on the first call made while
+// that context is current, and cached under the context's unique id: a
+// context created later (after cudaDeviceReset, or a separate driver-API
+// context) never reuses an address looked up for another one.  That first
+// call may also make the CUDA runtime load the library's device code into the
+// context (lazy loading), and loading code allocates device memory inside the
+// driver; this file itself calls no allocating routine.  Make the first call
+// in each context before any stream capture.  All calls in one context share
+// the one array, so calls that overlap on the GPU (different streams, or
+// different host threads without ordering) race on it; serialise them.  The
+// counts are fully rewritten by every call (nothing in the array has to start
+// at zero).
 #include <mutex>
 
 #include "../../include/ultratex.h"
@@ -32,24 +39,66 @@ constexpr int kNoAllocCounts = 1024;
 static __device__ __align__(256) int32_t g_compact_scratch[kNoAllocCounts];
 
 namespace {
-constexpr int kMaxDevices = 64;
-std::mutex g_setup_mutex;
-void* g_scratch_addr[kMaxDevices] = {};
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
 
-// Device address of g_compact_scratch on the current device (set up once).
+// Driver entry points, resolved once through the runtime (the library links
+// the static runtime only).
+template <typename F>
+F driver_fn(const char* name) {
+  void* p = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPoint(name, &p, cudaEnableDefault, &q) != cudaSuccess || q != cudaDriverEntryPointSuccess)
+    return nullptr;
+  return reinterpret_cast<F>(p);
+}
+
+constexpr int kMaxContexts = 64;
+struct ScratchEntry {
+  unsigned long long ctx_id;  // 0 = unused (driver context ids start at 1)
+  void* addr;
+};
+std::mutex g_setup_mutex;
+ScratchEntry g_scratch[kMaxContexts] = {};
+
+// Id of the current context; 0 if none is current or the query fails.
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_current = driver_fn<CtxGetCurrentFn>("cuCtxGetCurrent");
+  static CtxGetIdFn get_id = driver_fn<CtxGetIdFn>("cuCtxGetId");
+  if (!get_current || !get_id) return 0;
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (get_current(&ctx) != CUDA_SUCCESS || !ctx) return 0;
+  if (get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// Device address of g_compact_scratch in the current context.
 cudaError_t scratch_address(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  unsigned long long id = current_context_id();
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_compact_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = p;
+  if (id != 0) {
+    for (const ScratchEntry& e : g_scratch)
+      if (e.ctx_id == id) {
+        *out = e.addr;
+        return cudaSuccess;
+      }
   }
-  *out = g_scratch_addr[dev];
+  // first call in this context (the lookup also makes the runtime bind its
+  // context when none was current yet, so the id is taken again afterwards)
+  void* p = nullptr;
+  cudaError_t e = cudaGetSymbolAddress(&p, g_compact_scratch);
+  if (e != cudaSuccess) return e;
+  if (id == 0) id = current_context_id();
+  if (id != 0) {
+    for (ScratchEntry& s : g_scratch)
+      if (s.ctx_id == 0) {
+        s.ctx_id = id;
+        s.addr = p;
+        break;
+      }  // a full table only means later calls in this context look up again
+  }
+  *out = p;
   return cudaSuccess;
 }
 }  // namespace

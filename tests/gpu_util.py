@@ -52,3 +52,37 @@ def bits(t: torch.Tensor) -> np.ndarray:
     if t.dtype == torch.float32:
         return t.view(torch.int32).numpy()
     return t.numpy()
+
+
+def compare_topk_lists(rp, ci, rrp, rci, scores, kr):
+    """GPU Top-K lists (rp, ci) against the oracle's (rrp, rci): equal row
+    pointers; every row equal, except rows whose oracle K-th and (K+1)-th
+    scores lie within 1e-4 * max|s| (reading A16), where only near-tied blocks
+    may differ.  Returns the number of such near-tie rows."""
+    H, nq, nk = scores.shape
+    rp = np.asarray(rp)[:H * nq + 1]
+    assert np.array_equal(rp, rrp)
+    n_tie_rows = 0
+    for r in range(H * nq):
+        got = np.asarray(ci[rp[r]:rp[r + 1]])
+        want = rci[rrp[r]:rrp[r + 1]]
+        assert np.all(np.diff(got) > 0)
+        if np.array_equal(got, want):
+            continue
+        h, i = divmod(r, nq)
+        s = scores[h, i]
+        srt = np.sort(s)[::-1]
+        kth = srt[kr - 1]
+        eps = 1e-4 * np.abs(s).max()
+        assert kr < nk and srt[kr - 1] - srt[kr] < eps, f"row {r} differs without a near tie"
+        assert np.all(s[got] >= kth - eps)
+        n_tie_rows += 1
+    return n_tie_rows
+
+
+def head_lists(rp, ci, h, nq):
+    """The CSR rows of head h alone (row pointers rebased to 0)."""
+    rp = np.asarray(rp)
+    base = int(rp[h * nq])
+    end = int(rp[(h + 1) * nq])
+    return (rp[h * nq:(h + 1) * nq + 1] - base).astype(np.int64), np.asarray(ci[base:end])

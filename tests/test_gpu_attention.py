@@ -1,8 +1,11 @@
 """GPU parity: block-sparse attention forward and backward against the fp64 oracle.
 
-Small configurations are compared element by element in full; the 1024 and
-2048 canvases, in the launch configuration the benchmark times, are compared
-on seeded row samples that the oracle computes one by one.
+Small configurations, the 512 canvas and the whole 1024 canvas (24 heads,
+forward and backward, through the benchmark's path) are compared element by
+element in full.  The 2048 canvas, in the launch configuration the benchmark
+times, is compared on seeded row samples in every head plus two whole heads
+(dQ, dK, dV of every row); its Top-K lists are first checked against the
+oracle's own, and the oracle reference is computed from the oracle's lists.
 """
 import math
 
@@ -11,7 +14,7 @@ import pytest
 import torch
 
 import oracle.ultratex_oracle as o
-from gpu_util import assert_bf16_close, assert_f32_close, need_gpu, to_np
+from gpu_util import assert_bf16_close, assert_f32_close, compare_topk_lists, head_lists, need_gpu, to_np
 from synth import CONFIGS
 
 pytestmark = pytest.mark.gpu
@@ -122,45 +125,59 @@ def test_fwd_bf16_c512_full():
     assert np.abs(to_np(L) - rL).max() < 1e-3
 
 
-def _sampled_fwd_check(w, mode):
-    """Full-size problem through the bench's path; the oracle checks sampled rows."""
+def _chain(w, mode, backward):
+    """One pass of the whole hot path (compaction, lists, forward, backward,
+    scatter) through the benchmark's HotPath on the full-size canvas.  Returns
+    the device results, the canvas positions, the compacted inputs (fp32, the
+    exact bf16 values) and the block lists the oracle reference uses: the
+    bitmap's CSR, or the oracle's own Top-K lists after checking that the
+    GPU's lists equal them (rows with an A16 near tie may swap near-tied
+    blocks; if any such row exists the reference follows the GPU's lists)."""
     from paper_2609_23169_gb300 import path as P
     mask = w.canvas_mask()
     q, k, v = w.q(), w.k(), w.v()
+    do = w.dout() if backward else None
     bm = w.block_bitmap() if mode == "bitmap" else None
-    out = P.run_path(w, mask, q, k, v, None, bitmap=bm)
+    out = P.run_path(w, mask, q, k, v, do, bitmap=bm)
     idx = np.flatnonzero(mask)
+    assert out["N"] == len(idx) == w.N
+    assert np.array_equal(out["idx"].cpu().numpy(), idx)
     t = torch.from_numpy(idx)
-    qc, kc, vc = (x[t].float().numpy() for x in (q, k, v))
+    xs = [x[t].float().numpy() for x in ((q, k, v, do) if backward else (q, k, v))]
     nq = -(-w.N // w.block)
     rp = out["row_ptr"][:w.heads * nq + 1].cpu().numpy()
     ci = out["col_idx"][:int(rp[-1])].cpu().numpy()
     if mode == "bitmap":
         rrp, rci = o.bitmap_to_csr(bm)
-        assert np.array_equal(rp, rrp) and np.array_equal(ci[:len(rci)], rci)
-    rows = w.row_subsample(w.N, 0.01)
-    O = out["oc"].float().cpu().numpy()
-    L = out["lse"].cpu().numpy()
-    errs = []
-    for h in range(w.heads):
-        rO, rL = o.bsattn_fwd_rows(qc, kc, vc, rp, ci, w.block, h, rows)
-        errs.append((O[rows, h], rO))
-        assert np.abs(L[h, rows] - rL).max() < 1e-3
-    got = np.concatenate([e[0] for e in errs])
-    ref = np.concatenate([e[1] for e in errs])
-    s = assert_bf16_close(got, ref, w.name)
-    # scatter put the compacted rows at their canvas positions
-    oc = out["o_canvas"][torch.from_numpy(idx[rows]).cuda()].float().cpu().numpy()
-    assert np.array_equal(oc, O[rows])
-    return s
-
-
-def test_fwd_c1024_sampled():
-    print(_sampled_fwd_check(CONFIGS["c1024"], "bitmap"))
+        assert np.array_equal(rp, rrp) and np.array_equal(ci, rci)
+        n_ties = 0
+    else:
+        rrp, rci, scores, kr = o.topk_block_mask(xs[0], xs[1], w.block, w.rho)
+        n_ties = compare_topk_lists(rp, ci, rrp, rci, scores, kr)
+        print(f"{w.name}: Top-K near-tie rows {n_ties} of {w.heads * nq}")
+        if n_ties:
+            rrp, rci = rp, ci
+    return out, idx, xs, rrp, rci
 
 
 def test_fwd_c2048_sampled():
-    print(_sampled_fwd_check(CONFIGS["c2048"], "topk"))
+    """2048 canvas, Top-K rho = 0.12: the lists against the oracle's, then O and
+    LSE of a seeded 1% of query rows in every head against the oracle computed
+    from the oracle's lists; the scatter put those rows at their positions."""
+    w = CONFIGS["c2048"]
+    out, idx, (qc, kc, vc), rp, ci = _chain(w, "topk", backward=False)
+    rows = w.row_subsample(w.N, 0.01)
+    O = out["oc"].float().cpu().numpy()
+    L = out["lse"].cpu().numpy()
+    got, ref = [], []
+    for h in range(w.heads):
+        rO, rL = o.bsattn_fwd_rows(qc, kc, vc, rp, ci, w.block, h, rows)
+        got.append(O[rows, h])
+        ref.append(rO)
+        assert np.abs(L[h, rows] - rL).max() < 1e-3
+    print(assert_bf16_close(np.concatenate(got), np.concatenate(ref), w.name))
+    oc = out["o_canvas"][torch.from_numpy(idx[rows]).cuda()].float().cpu().numpy()
+    assert np.array_equal(oc, O[rows])
 
 
 # ----------------------------------------------------------------- backward
@@ -197,8 +214,9 @@ def test_bwd_bf16_small_full(N, H, d, dens, seed):
         assert_bf16_close(to_np(g), r, name)
 
 
-def test_bwd_c512_four_heads_full():
-    w = CONFIGS["c512"].with_(heads=4)
+def test_bwd_c512_full():
+    """The 512 canvas, all 24 heads, forward and backward in full."""
+    w = CONFIGS["c512"]
     idx = torch.from_numpy(np.flatnonzero(w.canvas_mask()))
     q, k, v, do = (x[idx] for x in (w.q(), w.k(), w.v(), w.dout()))
     bm = w.block_bitmap()
@@ -209,20 +227,45 @@ def test_bwd_c512_four_heads_full():
         print(name, assert_bf16_close(to_np(g), r, name))
 
 
-def _sampled_bwd_check(w, mode, key_heads=(0, 7)):
-    """Full-size forward + backward through the bench's path; sampled dQ rows in
-    every head and sampled dK/dV rows in two heads against the oracle."""
-    from paper_2609_23169_gb300 import path as P
-    mask = w.canvas_mask()
-    q, k, v, do = w.q(), w.k(), w.v(), w.dout()
-    bm = w.block_bitmap() if mode == "bitmap" else None
-    out = P.run_path(w, mask, q, k, v, do, bitmap=bm)
-    idx = np.flatnonzero(mask)
-    t = torch.from_numpy(idx)
-    qc, kc, vc, dc = (x[t].float().numpy() for x in (q, k, v, do))
+def _check_scatter(out, idx, mask, rows):
+    """KEEP put O at the canvas positions; ZERO put the gradients there and
+    zeros on every background row."""
+    at = torch.from_numpy(idx[rows]).cuda()
+    assert torch.equal(out["o_canvas"][at], out["oc"][torch.from_numpy(rows).cuda()])
+    bg = torch.from_numpy(np.flatnonzero(mask == 0)).cuda()
+    for name, comp in (("dq_canvas", "dqc"), ("dk_canvas", "dkc"), ("dv_canvas", "dvc")):
+        g = out[name]
+        assert torch.equal(g[at], out[comp][torch.from_numpy(rows).cuda()])
+        assert torch.all(g[bg] == 0)
+
+
+def test_fwd_bwd_c1024_full():
+    """The whole 1024 canvas (N = 23,959, 24 heads, structured lists, density
+    ~0.24) through the benchmark's path: O, LSE, dQ, dK and dV of every row and
+    head against the full oracle, element by element."""
+    w = CONFIGS["c1024"]
+    out, idx, (qc, kc, vc, dc), rp, ci = _chain(w, "bitmap", backward=True)
+    rO, rL = o.bsattn_fwd(qc, kc, vc, rp, ci, w.block)
+    print("O c1024", assert_bf16_close(to_np(out["oc"]), rO, "O c1024"))
+    L = out["lse"].cpu().numpy()
+    fin = np.isfinite(rL)
+    assert np.array_equal(np.isfinite(L), fin)
+    assert np.abs(L[fin] - rL[fin]).max() < 1e-3
+    rq, rk, rv = o.bsattn_bwd(qc, kc, vc, dc, rp, ci, w.block)
+    for name, comp, r in (("dQ", "dqc", rq), ("dK", "dkc", rk), ("dV", "dvc", rv)):
+        print(name, "c1024", assert_bf16_close(to_np(out[comp]), r, name + " c1024"))
+    _check_scatter(out, idx, w.canvas_mask(), np.arange(0, w.N, 37))
+
+
+def test_bwd_c2048():
+    """2048 canvas, Top-K rho = 0.12, forward + backward through the
+    benchmark's path: dQ of a seeded 0.5% of query rows in every head, and
+    dQ, dK, dV of every row of two whole heads (the first and the last, which
+    the backward hands out first and last), against the oracle computed from
+    the oracle's own lists."""
+    w = CONFIGS["c2048"]
+    out, idx, (qc, kc, vc, dc), rp, ci = _chain(w, "topk", backward=True)
     nq = -(-w.N // w.block)
-    rp = out["row_ptr"][:w.heads * nq + 1].cpu().numpy()
-    ci = out["col_idx"][:int(rp[-1])].cpu().numpy()
     rows = w.row_subsample(w.N, 0.005)
     dq = out["dqc"].float().cpu().numpy()
     dk = out["dkc"].float().cpu().numpy()
@@ -231,28 +274,14 @@ def _sampled_bwd_check(w, mode, key_heads=(0, 7)):
     for h in range(w.heads):
         got.append(dq[rows, h])
         ref.append(o.bsattn_bwd_dq_rows(qc, kc, vc, dc, rp, ci, w.block, h, rows))
-    sq = assert_bf16_close(np.concatenate(got), np.concatenate(ref), "dQ " + w.name)
-    krows = rows[:24]
-    gk, gv, rk, rv = [], [], [], []
-    for h in key_heads:
-        a, b = o.bsattn_bwd_dkdv_rows(qc, kc, vc, dc, rp, ci, w.block, h, krows)
-        gk.append(dk[krows, h]); gv.append(dv[krows, h]); rk.append(a); rv.append(b)
-    sk = assert_bf16_close(np.concatenate(gk), np.concatenate(rk), "dK " + w.name)
-    sv = assert_bf16_close(np.concatenate(gv), np.concatenate(rv), "dV " + w.name)
-    # scatter (ZERO mode) put gradients at canvas positions and zeros elsewhere
-    gq = out["dq_canvas"]
-    assert torch.equal(gq[torch.from_numpy(idx[rows]).cuda()].float().cpu(), torch.from_numpy(dq[rows]))
-    bg = torch.from_numpy(np.flatnonzero(mask == 0)[:1000]).cuda()
-    assert torch.all(gq[bg] == 0)
-    return sq, sk, sv
-
-
-def test_bwd_c1024_sampled():
-    print(_sampled_bwd_check(CONFIGS["c1024"], "bitmap"))
-
-
-def test_bwd_c2048_sampled():
-    print(_sampled_bwd_check(CONFIGS["c2048"], "topk"))
+    print("dQ rows c2048", assert_bf16_close(np.concatenate(got), np.concatenate(ref), "dQ rows c2048"))
+    for h in (0, w.heads - 1):
+        hr, hc = head_lists(rp, ci, h, nq)
+        sl = slice(h, h + 1)
+        rq, rk, rv = o.bsattn_bwd(qc[:, sl], kc[:, sl], vc[:, sl], dc[:, sl], hr, hc, w.block)
+        for name, g, r in (("dQ", dq, rq), ("dK", dk, rk), ("dV", dv, rv)):
+            print(name, "c2048 head", h, assert_bf16_close(g[:, sl], r, f"{name} c2048 head {h}"))
+    _check_scatter(out, idx, w.canvas_mask(), rows)
 
 
 def test_hot_path_count_in_pinned_or_device_memory():

@@ -4,7 +4,7 @@ import pytest
 import torch
 
 import oracle.ultratex_oracle as o
-from gpu_util import bits, need_gpu
+from gpu_util import bits, compare_topk_lists, need_gpu
 from synth import CONFIGS
 
 pytestmark = pytest.mark.gpu
@@ -193,24 +193,8 @@ def _check_topk(qc_np, kc_np, rp, ci, cp, ri, b, rho, allow_near_ties=False):
     scores are within 1e-4*max|s| may differ, but only by swapping near-tied blocks."""
     rrp, rci, scores, kr = o.topk_block_mask(qc_np, kc_np, b, rho)
     H, nq, _ = scores.shape
-    assert np.array_equal(rp, rrp)
-    n_tie_rows = 0
-    for r in range(H * nq):
-        got = ci[rp[r]:rp[r + 1]]
-        want = rci[rrp[r]:rrp[r + 1]]
-        assert np.all(np.diff(got) > 0)
-        if np.array_equal(got, want):
-            continue
-        assert allow_near_ties, f"row {r}: {got} != {want}"
-        h, i = divmod(r, nq)
-        s = scores[h, i]
-        srt = np.sort(s)[::-1]
-        kth = srt[kr - 1]
-        eps = 1e-4 * np.abs(s).max()
-        assert kr < nq and srt[kr - 1] - srt[kr] < eps, f"row {r} differs without a near tie"
-        # every chosen block is within eps of the threshold or above it
-        assert np.all(s[got] >= kth - eps)
-        n_tie_rows += 1
+    n_tie_rows = compare_topk_lists(rp, ci, rrp, rci, scores, kr)
+    assert allow_near_ties or n_tie_rows == 0
     rcp, rri = o.csr_to_csc(rp, ci, H, nq, nq)   # transpose of the GPU's own lists
     assert np.array_equal(cp, rcp) and np.array_equal(ri[:len(rri)], rri)
     return n_tie_rows
