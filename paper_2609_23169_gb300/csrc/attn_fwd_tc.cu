@@ -9,16 +9,24 @@
 //               128B-swizzled shared tiles.  A K stage is released by the MMA
 //               that consumed it (S = Q K^T), a V stage by O += P V.
 //   warp 1      TMEM owner and MMA issuer (one elected thread):
-//               S_t = Q K_t^T (both operands in shared memory) into one of two
-//               TMEM S buffers, then O += P_{t-1} V_{t-1} with P read from TMEM
-//               (only V is read from shared memory).
-//   warps 2-5   softmax: thread = query row = TMEM lane.  Reads S_t from TMEM,
-//               masks the ragged last key block, keeps a running row maximum
-//               (rescaling O in TMEM only when the maximum grew by more than
-//               2^8, so the exponentials stay bounded), writes P_t as bf16
-//               pairs into a TMEM P buffer, and finally normalises O and
-//               writes O (bf16) and LSE (fp32, natural log).
-// TMEM columns: S0 [0,128), S1 [128,256), O [256,256+D), P0 [384,448), P1 [448,512).
+//               S_t = Q K_t^T with Q read from TMEM (only K from shared
+//               memory) into one of two TMEM S buffers, two key blocks ahead
+//               of O += P_u V_u with P also read from TMEM (only V from shared
+//               memory).
+//   warps 2-5   softmax: thread = query row = TMEM lane.  At the start of an
+//               item they copy its Q tile from shared memory into TMEM (the A
+//               operand of S), then finish the previous item (normalise O,
+//               write O in bf16 and LSE in fp32, natural log) while the tensor
+//               core already computes the new item's first S blocks.  Per key
+//               block: read S_t from TMEM, mask the ragged last key block, keep
+//               a running row maximum (rescaling O in TMEM only when the
+//               maximum grew by more than 2^8, so the exponentials stay
+//               bounded), write P_t as bf16 pairs into the TMEM P buffer.
+// Reading Q from TMEM halves the shared-memory operand traffic of S = Q K^T;
+// per key block the shared memory then serves K and V to the tensor core and
+// their TMA writes (128 KB), about what the two 128 x 128 x 128 products take.
+// TMEM columns: S0 [0,128), S1 [128,256), O [256,256+D), P [384,448),
+// Q [448,448+D/2).
 // Blocks of 64 rows (b_q or b_kv) are served by the same 128 x 128 tiles: an
 // item's fine key-block lists are merged into 128-row key tiles with a mask of
 // the listed 64 x 64 sub-blocks (TileList), and the softmax sets the scores of
@@ -36,7 +44,7 @@ constexpr int kBN = 128;  // key rows per tile
 constexpr int kFwdThreads = 192;
 constexpr int kStages = 3;                       // K and V ring depth
 constexpr uint32_t kTileChunkBytes = 128 * 128;  // 128 rows x 128 bytes (64 bf16)
-constexpr uint32_t kColO = 256, kColP = 384;     // TMEM column bases
+constexpr uint32_t kColO = 256, kColP = 384, kColQ = 448;  // TMEM column bases
 
 template <int D>
 struct FwdSmem {
@@ -46,10 +54,11 @@ struct FwdSmem {
   alignas(1024) uint8_t q[kQBytes];
   alignas(1024) uint8_t k[kStages][kKVBytes];
   alignas(1024) uint8_t v[kStages][kKVBytes];
-  uint64_t q_full, q_empty;
+  uint64_t q_full, q_empty;    // shared Q tile: TMA landed / copied into TMEM
+  uint64_t qt_full, qt_empty;  // TMEM Q: written by the softmax warps / last S of the item done
   uint64_t k_full[kStages], v_full[kStages], k_empty[kStages], v_empty[kStages];
   uint64_t s_full[2], s_empty[2];
-  uint64_t p_full[2], pv_done[2];
+  uint64_t p_full, pv_done;    // one TMEM P buffer
   uint64_t o_empty, mma_done;
   uint32_t tmem_base;
   int abort_flag;
@@ -85,7 +94,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.q_full, 1);
-    mbar_init(&sm.q_empty, 1);
+    mbar_init(&sm.q_empty, 4);
+    mbar_init(&sm.qt_full, 4);
+    mbar_init(&sm.qt_empty, 1);
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.k_full[s], 1);
       mbar_init(&sm.v_full[s], 1);
@@ -95,9 +106,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     for (int s = 0; s < 2; ++s) {
       mbar_init(&sm.s_full[s], 1);
       mbar_init(&sm.s_empty[s], 4);
-      mbar_init(&sm.p_full[s], 4);
-      mbar_init(&sm.pv_done[s], 1);
     }
+    mbar_init(&sm.p_full, 4);
+    mbar_init(&sm.pv_done, 1);
     mbar_init(&sm.o_empty, 4);
     mbar_init(&sm.mma_done, 1);
     sm.abort_flag = 0;
@@ -172,7 +183,6 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN, false, false);
       constexpr uint32_t idesc_o = idesc_bf16_f32(kBM, D, false, true);
-      const uint32_t q_addr = smem_u32(sm.q);
       uint32_t qi = 0, oi = 0, kv0 = 0, sc0 = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
@@ -181,7 +191,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
                 prm.list_shift);
         const int L = tl.count_warp();
         if (L <= 0) continue;
-        if (!(ok = warp_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        // Q of this item in TMEM (the softmax warps copied it there)
+        if (!(ok = warp_wait(&sm.qt_full, qi & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         // S runs two key blocks ahead of P V: S_{u+2} goes into the S buffer
         // that softmax u has just read, so the tensor core computes it while
         // the softmax works, and PV_u follows as soon as P_u is in TMEM.
@@ -195,27 +206,27 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint32_t off = (kk >> 2) * kTileChunkBytes + (kk & 3) * 32;
-            mma_bf16_ss_w(tmem + sb * 128, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024),
-                          idesc_s, kk > 0);
+            mma_bf16_ts_w(tmem + sb * 128, tmem + kColQ + kk * 8, sdesc_sw128(k_addr + off, 16, 1024), idesc_s,
+                          kk > 0);
           }
           mma_commit_w(&sm.s_full[sb]);
           mma_commit_w(&sm.k_empty[st]);
-          if (t == L - 1) mma_commit_w(&sm.q_empty);
+          if (t == L - 1) mma_commit_w(&sm.qt_empty);  // Q's TMEM columns are free once these S are done
           return true;
         };
         auto issue_pv = [&](int u) -> bool {
           const uint32_t kv = kv0 + u, st = kv % kStages, n = kv / kStages;
-          const uint32_t sc = sc0 + u, pb = sc & 1, np = sc >> 1;
-          if (!warp_wait(&sm.p_full[pb], np & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+          const uint32_t sc = sc0 + u;
+          if (!warp_wait(&sm.p_full, sc & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
           if (!warp_wait(&sm.v_full[st], n & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
           if (u == 0 && !warp_wait(&sm.o_empty, (oi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)) return false;
           tc_fence_after();
           const uint32_t v_addr = smem_u32(sm.v[st]);
 #pragma unroll
           for (int kk = 0; kk < kBN / 16; ++kk)
-            mma_bf16_ts_w(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
-                          sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024), idesc_o, (u > 0 || kk > 0));
-          mma_commit_w(&sm.pv_done[pb]);
+            mma_bf16_ts_w(tmem + kColO, tmem + kColP + kk * 8, sdesc_sw128(v_addr + kk * 2048, kTileChunkBytes, 1024),
+                          idesc_o, (u > 0 || kk > 0));
+          mma_commit_w(&sm.pv_done);
           mma_commit_w(&sm.v_empty[st]);
           return true;
         };
@@ -239,28 +250,97 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     const uint32_t row = quarter * 32 + lane;
     const uint32_t lane_base = (quarter * 32) << 16;
     const float c = prm.scale_log2;
-    uint32_t sc0 = 0;
+    uint32_t sc0 = 0, qi = 0;
     bool ok = true;
     const uint32_t rh = row >> 6;  // which 64-row half of the query tile
+    // Q tile of the next item: shared memory (128B-swizzled, as TMA wrote it)
+    // -> registers -> TMEM, this thread's row, bf16 pairs (element 2u in the
+    // low half of column u), the A-operand layout of S = Q K^T.
+    auto load_q = [&]() -> bool {
+      if (!warp_wait(&sm.q_full, qi & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+      if (!warp_wait(&sm.qt_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int cc = 0; cc < C; ++cc) {
+        uint32_t qv[32];
+        const uint32_t base = smem_u32(sm.q) + cc * kTileChunkBytes + row * 128;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                       : "=r"(qv[4 * u]), "=r"(qv[4 * u + 1]), "=r"(qv[4 * u + 2]), "=r"(qv[4 * u + 3])
+                       : "r"(base + ((u ^ (row & 7)) << 4)));
+        tmem_st32(tmem + lane_base + kColQ + cc * 32, qv);
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&sm.qt_full);
+        mbar_arrive(&sm.q_empty);
+      }
+      ++qi;
+      return true;
+    };
+    // The previous item's epilogue (O / l -> bf16, LSE) runs after the next
+    // item's Q is in TMEM, so the tensor core computes the next S blocks
+    // meanwhile.
+    bool pend = false;
+    float e_m = 0.f, e_l = 0.f;
+    uint32_t e_last = 0;
+    int64_t e_grow = 0;
+    int e_h = 0;
+    auto epilogue = [&]() -> bool {
+      if (!warp_wait(&sm.pv_done, e_last & 1, abort_flag, prm.status, prm.timeout_ns)) return false;
+      tc_fence_after();
+      const bool row_ok = e_grow < prm.N;
+      __nv_bfloat16* orow = prm.o + e_grow * prm.rs + (int64_t)e_h * D;
+      const float inv = (!kSub || e_l > 0.f) ? 1.0f / e_l : 0.f;  // a row that saw no key: O = 0, LSE = -inf
+#pragma unroll
+      for (int g = 0; g < D / 32; ++g) {
+        uint32_t r[32];
+        tmem_ld32(tmem + lane_base + kColO + g * 32, r);
+        tmem_wait_ld();
+        if (row_ok) {
+#pragma unroll
+          for (int x = 0; x < 32; x += 8) {
+            uint4 v;
+            v.x = pack_bf16x2(__uint_as_float(r[x + 0]) * inv, __uint_as_float(r[x + 1]) * inv);
+            v.y = pack_bf16x2(__uint_as_float(r[x + 2]) * inv, __uint_as_float(r[x + 3]) * inv);
+            v.z = pack_bf16x2(__uint_as_float(r[x + 4]) * inv, __uint_as_float(r[x + 5]) * inv);
+            v.w = pack_bf16x2(__uint_as_float(r[x + 6]) * inv, __uint_as_float(r[x + 7]) * inv);
+            *reinterpret_cast<uint4*>(orow + g * 32 + x) = v;
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.o_empty);
+      if (row_ok)
+        prm.lse[(int64_t)e_h * prm.N + e_grow] =
+            (!kSub || e_l > 0.f) ? (e_m + log2f(e_l)) * 0.69314718055994531f : -INFINITY;
+      return true;
+    };
     for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
       const int h = w / prm.nq, i = w % prm.nq;
       TileList<kSub> tl;
       tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
       const int L = tl.count_warp();
       const int64_t grow = (int64_t)i * kBM + row;
-      const bool row_ok = grow < prm.N;
-      __nv_bfloat16* orow = prm.o + grow * prm.rs + (int64_t)h * D;
       if (L <= 0) {
-        if (row_ok) {
+        if (grow < prm.N) {
+          __nv_bfloat16* orow = prm.o + grow * prm.rs + (int64_t)h * D;
           for (int e = 0; e < D; e += 8) *reinterpret_cast<uint4*>(orow + e) = make_uint4(0, 0, 0, 0);
           prm.lse[(int64_t)h * prm.N + grow] = -INFINITY;
         }
         continue;
       }
+      if (!(ok = load_q())) break;
+      if (pend && !(ok = epilogue())) break;
+      pend = false;
       float m_used = 0.f, l = 0.f;
       int j_next = 0;
       uint32_t bits_next = 0;
-      if (L > 0) tl.next(j_next, bits_next);
+      tl.next(j_next, bits_next);
       for (int t = 0; t < L; ++t) {
         const int j = j_next;
         const uint32_t bits = bits_next;
@@ -315,9 +395,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         } else {
           const bool need = mx > m_used + 8.0f;
           if (__any_sync(0xffffffffu, need)) {
-            const uint32_t pc = sc - 1;
-            if (!(ok = warp_wait(&sm.pv_done[pc & 1], (pc >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
-              break;
+            // O holds P V up to the previous key block once that MMA finished
+            if (!(ok = warp_wait(&sm.pv_done, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             tc_fence_after();
             const float alpha = need ? ex2_approx(m_used - mx) : 1.0f;
 #pragma unroll
@@ -355,47 +434,26 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           }
         }
         l += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
-        // the TMEM P buffer is free once the P V MMA of its previous use finished
-        if (!(ok = warp_wait(&sm.pv_done[sb], (ns & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
+        // the TMEM P buffer is free once the previous key block's P V finished
+        if (!(ok = warp_wait(&sm.pv_done, (sc & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
-        tmem_st32(tmem + lane_base + kColP + sb * 64, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
-        tmem_st32(tmem + lane_base + kColP + sb * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[32]));
+        tmem_st32(tmem + lane_base + kColP, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
+        tmem_st32(tmem + lane_base + kColP + 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[32]));
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.p_full[sb]);
+        if (lane == 0) mbar_arrive(&sm.p_full);
       }
       if (!ok) break;
-      // epilogue: O / l -> bf16, LSE
-      const uint32_t last = sc0 + L - 1;
-      if (!(ok = warp_wait(&sm.pv_done[last & 1], (last >> 1) & 1, abort_flag, prm.status, prm.timeout_ns))) break;
-      tc_fence_after();
-      const float inv = (!kSub || l > 0.f) ? 1.0f / l : 0.f;  // a row that saw no key: O = 0, LSE = -inf
-#pragma unroll
-      for (int g = 0; g < D / 32; ++g) {
-        uint32_t r[32];
-        tmem_ld32(tmem + lane_base + kColO + g * 32, r);
-        tmem_wait_ld();
-        if (row_ok) {
-#pragma unroll
-          for (int x = 0; x < 32; x += 8) {
-            uint4 v;
-            v.x = pack_bf16x2(__uint_as_float(r[x + 0]) * inv, __uint_as_float(r[x + 1]) * inv);
-            v.y = pack_bf16x2(__uint_as_float(r[x + 2]) * inv, __uint_as_float(r[x + 3]) * inv);
-            v.z = pack_bf16x2(__uint_as_float(r[x + 4]) * inv, __uint_as_float(r[x + 5]) * inv);
-            v.w = pack_bf16x2(__uint_as_float(r[x + 6]) * inv, __uint_as_float(r[x + 7]) * inv);
-            *reinterpret_cast<uint4*>(orow + g * 32 + x) = v;
-          }
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.o_empty);
-      if (row_ok)
-        prm.lse[(int64_t)h * prm.N + grow] =
-            (!kSub || l > 0.f) ? (m_used + log2f(l)) * 0.69314718055994531f : -INFINITY;
+      pend = true;
+      e_m = m_used;
+      e_l = l;
+      e_last = sc0 + L - 1;
+      e_grow = grow;
+      e_h = h;
       sc0 += L;
     }
+    if (ok && pend) ok = epilogue();
   }
 
   tc_fence_before();
