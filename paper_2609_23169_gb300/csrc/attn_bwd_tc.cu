@@ -14,9 +14,17 @@
 //                           fp32 accumulator (below).
 //   bwd_dq_finalize_kernel  dQ = scale * accumulator, bf16.
 //
-// Blocks of 64 rows (b_q or b_kv) are served by the same 128 x 128 tiles: the
-// item's fine lists are merged into 128-row query tiles with a mask of the
-// listed 64 x 64 sub-blocks (TileList); P of unlisted sub-blocks is zero.
+// Blocks of 64 rows (b_q or b_kv) are served by the same 128 x 128 tiles:
+//   b_q = 64:   two listed 64-row query blocks fill one 128-row query tile
+//               (Q and dO loaded as two 64-row TMA boxes, PairList):
+//               consecutive entries of the key block's list for b_kv = 128
+//               (nothing discarded), the two 64-row key blocks' lists in
+//               lockstep for b_kv = 64 (key rows 0-63 see the low half of the
+//               query tile, key rows 64-127 the high half); the dQ^T drain
+//               adds each half into its own query block;
+//   b_q = 128, b_kv = 64:  the item's two lists are merged into 128-row query
+//               tiles with a mask of the listed 64 x 64 sub-blocks (TileList).
+// P of the sub-blocks a key row does not see is zero.
 // All waits are bounded (UT_ERR_TIMEOUT on expiry, then drain and return).
 #include "common.cuh"
 #include "kernels.h"
@@ -159,11 +167,34 @@ UT_DEV void red_add_f32(float* p, float v) {
   asm volatile("red.relaxed.gpu.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
 }
 
-template <int D, bool kSub>
+// The query steps of an item.  kMode 0: 128-row blocks on both sides; 1:
+// 128-row query blocks, 64-row key blocks (merged lists, TileList); 2: 64-row
+// query blocks paired into 128-row tiles (PairList).  next() gives the tile's
+// query blocks (mode 2: the 64-row blocks of the low and high halves, -1 if
+// missing; otherwise lo = the 128-row query tile) and the visibility bits.
+template <int kMode>
+struct QuerySteps {
+  TileList<kMode == 1> tl;
+  PairList pl;
+  UT_DEV void init(const BwdParams& prm, int h, int j) {
+    if (kMode == 2) pl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile == 2);
+    else tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+  }
+  UT_DEV int count_warp() const { return kMode == 2 ? pl.count() : tl.count_warp(); }
+  UT_DEV bool empty() const { return kMode == 2 ? pl.empty() : tl.empty(); }
+  UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
+    if (kMode == 2) return pl.next(lo, hi, bits);
+    hi = -1;
+    return tl.next(lo, bits);
+  }
+};
+
+template <int D, int kMode>
 __global__ void __launch_bounds__(kFuThreads, 1)
     bwd_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
                      const BwdParams prm, float* __restrict__ dq_acc) {
+  constexpr bool kSub = kMode != 0;  // 64-row blocks on at least one side
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   FusedSmem<D>& sm = *reinterpret_cast<FusedSmem<D>*>(smem_raw);
   constexpr int C = FusedSmem<D>::kC;
@@ -274,8 +305,8 @@ __global__ void __launch_bounds__(kFuThreads, 1)
           }
           if (w < 0) break;
           const int h = w / prm.nq, j = w % prm.nq;
-          TileList<kSub> tl;
-          tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+          QuerySteps<kMode> tl;
+          tl.init(prm, h, j);
           if (tl.empty()) continue;
           if (is_q) {
             if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -286,14 +317,23 @@ __global__ void __launch_bounds__(kFuThreads, 1)
             }
             ++ki;
           }
-          int i;
+          int i, ih;
           uint32_t bits;
-          for (; tl.next(i, bits); ++qd) {
+          for (; tl.next(i, ih, bits); ++qd) {
             const uint32_t st = qd % nst, n = qd / nst;
             if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             mbar_expect_tx(&full[st], TB);
-            for (int c = 0; c < C; ++c)
-              tma_load_2d(ring + st * TB + c * kChunk, tmap, &full[st], h * D + c * 64, i * kTile, pol_qd);
+            uint8_t* dst = ring + st * TB;
+            if (kMode == 2) {  // two 64-row boxes: rows 0-63 and 64-127 of each 128-row sub-tile
+              const int b0 = PairList::load_lo(i, ih), b1 = PairList::load_hi(i, ih);
+              for (int c = 0; c < C; ++c) {
+                tma_load_2d(dst + c * kChunk, tmap, &full[st], h * D + c * 64, b0 * 64, pol_qd);
+                tma_load_2d(dst + c * kChunk + 64 * 128, tmap, &full[st], h * D + c * 64, b1 * 64, pol_qd);
+              }
+            } else {
+              for (int c = 0; c < C; ++c)
+                tma_load_2d(dst + c * kChunk, tmap, &full[st], h * D + c * 64, i * kTile, pol_qd);
+            }
           }
           if (!ok) break;
         }
@@ -317,8 +357,8 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         for (;;) {
           int w;
           if (!(ok = next_item(kk, w, false)) || w < 0) break;
-          TileList<kSub> tl;
-          tl.init(prm.ptr, prm.idx, w / prm.nq, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+          QuerySteps<kMode> tl;
+          tl.init(prm, w / prm.nq, w % prm.nq);
           const int L = tl.count_warp();
           if (L <= 0) continue;
           if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -419,8 +459,8 @@ __global__ void __launch_bounds__(kFuThreads, 1)
       int w;
       if (!(ok = next_item(kk, w, false)) || w < 0) break;
       const int h = w / prm.nq, j = w % prm.nq;
-      TileList<kSub> tl;
-      tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+      QuerySteps<kMode> tl;
+      tl.init(prm, h, j);
       const int L = tl.count_warp();
       const int64_t gk = (int64_t)j * kTile + krow;
       const bool row_ok = gk < prm.N;
@@ -435,12 +475,18 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         continue;
       }
       // this thread's element of the query-row vectors (LSE*log2e for threads
-      // 0-127, D for 128-255) is loaded one pair ahead
-      const float* rv_src = (tid < kTile ? prm.lse2 + tid : prm.dsum + (tid - kTile)) + (int64_t)h * prm.Np;
-      int i_next;
+      // 0-127, D for 128-255) is loaded one pair ahead: query column
+      // tid mod 128 of the tile, in its 64-row half
+      const uint32_t qcol = tid & (kTile - 1), qhalf = qcol >> 6;
+      const float* rv_src = (tid < kTile ? prm.lse2 : prm.dsum) + (int64_t)h * prm.Np + (qcol & 63);
+      auto rv_row = [&](int lo, int hi) -> int64_t {  // first row of this thread's 64-row query half
+        if (kMode == 2) return 64 * (int64_t)(qhalf ? PairList::load_hi(lo, hi) : PairList::load_lo(lo, hi));
+        return (int64_t)lo * kTile + 64 * qhalf;
+      };
+      int i_next, ih_next;
       uint32_t bits_next;
-      tl.next(i_next, bits_next);
-      float rv = rv_src[(int64_t)i_next * kTile];
+      tl.next(i_next, ih_next, bits_next);
+      float rv = rv_src[rv_row(i_next, ih_next)];
       for (int t = 0; t < L; ++t) {
         const uint32_t qd = qd0 + t;
         // this half's 64 query columns and this thread's 64 key rows form one
@@ -452,7 +498,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         if (tid < kTile) sm.lse2[qd & 1][tid] = rv;
         else sm.dsum[qd & 1][tid - kTile] = rv;
         mbar_arrive(&sm.rowvec_full[qd & 1]);
-        if (t + 1 < L && tl.next(i_next, bits_next)) rv = rv_src[(int64_t)i_next * kTile];
+        if (t + 1 < L && tl.next(i_next, ih_next, bits_next)) rv = rv_src[rv_row(i_next, ih_next)];
         if (!(ok = warp_wait(&sm.rowvec_full[qd & 1], (qd >> 1) & 1, abort_flag, prm.status, prm.timeout_ns)))
           break;
         const float* ls = sm.lse2[qd & 1] + half * HC;
@@ -573,20 +619,25 @@ __global__ void __launch_bounds__(kFuThreads, 1)
       int w;
       if (!(ok = next_item(kk, w, false)) || w < 0) break;
       const int h = w / prm.nq;
-      TileList<kSub> tl;
-      tl.init(prm.ptr, prm.idx, h, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+      QuerySteps<kMode> tl;
+      tl.init(prm, h, w % prm.nq);
       const int L = tl.count_warp();
       if (L <= 0) continue;
       for (int t = 0; t < L; ++t) {
         const uint32_t qd = qd0 + t;
-        int i;
+        int i, ih;
         uint32_t bits;
-        tl.next(i, bits);
+        tl.next(i, ih, bits);
         if (!(ok = warp_wait(&sm.ds_done, qd & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
-        float* dst = dq_acc + (((int64_t)h * prm.Np + (int64_t)i * kTile) * D + dcol);
 #pragma unroll
         for (int g = 0; g < 2; ++g) {
+          // query half g of the tile: rows of 64-row block lo / hi (mode 2), or
+          // rows g * 64 .. of the 128-row query block; a missing block (-1)
+          // has dS^T = 0 there and is not added
+          const int blk = kMode == 2 ? (g ? ih : i) : 0;
+          const int64_t row0 = kMode == 2 ? 64 * (int64_t)blk : (int64_t)i * kTile + 64 * g;
+          float* dst = dq_acc + (((int64_t)h * prm.Np + row0) * D + dcol);
           uint32_t r[64];
           tmem_ld64(tmem + lane_base + kColRQ + g * 64, r);
           if (g == 1) {
@@ -594,9 +645,9 @@ __global__ void __launch_bounds__(kFuThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&sm.dq_empty);
           }
-          if (dcol < (uint32_t)D) {
+          if (dcol < (uint32_t)D && blk >= 0) {
 #pragma unroll
-            for (int x = 0; x < 64; ++x) red_add_f32(dst + (int64_t)(g * 64 + x) * D, __uint_as_float(r[x]));
+            for (int x = 0; x < 64; ++x) red_add_f32(dst + (int64_t)x * D, __uint_as_float(r[x]));
           }
         }
       }
@@ -639,22 +690,22 @@ size_t attn_bwd_tc_ws(const AttnProblem& p) {
 constexpr size_t kMaxDynSmem = 232448;  // 227 KB opt-in per block on sm_100/sm_103
 static_assert(sizeof(FusedSmem<128>) <= kMaxDynSmem, "fused backward shared layout exceeds the per-block limit");
 
-template <int D, bool kSub>
+template <int D, int kMode>
 static cudaError_t launch_bwd_fused(const AttnProblem& p, const CUtensorMap* tm, BwdParams prm, float* dq_acc,
                                    __nv_bfloat16* dq, int sms, cudaStream_t s) {
   const int n_items = prm.n_items;
   const int grid = n_items < sms ? n_items : sms;
   const size_t smem = sizeof(FusedSmem<D>);
   cudaError_t e =
-      cudaFuncSetAttribute(bwd_fused_kernel<D, kSub>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      cudaFuncSetAttribute(bwd_fused_kernel<D, kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   // the setmaxnreg split assumes exactly kFuRegLaunch registers per thread at
   // launch: with fewer, the increases would wait for registers that never come
   cudaFuncAttributes fa;
-  e = cudaFuncGetAttributes(&fa, bwd_fused_kernel<D, kSub>);
+  e = cudaFuncGetAttributes(&fa, bwd_fused_kernel<D, kMode>);
   if (e != cudaSuccess) return e;
   if (fa.numRegs != kFuRegLaunch) return cudaErrorInvalidConfiguration;
-  bwd_fused_kernel<D, kSub><<<grid, kFuThreads, smem, s>>>(tm[0], tm[1], tm[2], tm[3], prm, dq_acc);
+  bwd_fused_kernel<D, kMode><<<grid, kFuThreads, smem, s>>>(tm[0], tm[1], tm[2], tm[3], prm, dq_acc);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int64_t n8 = p.N * p.H * D / 8;
@@ -684,11 +735,16 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
       p.row_stride, lse2, dsum);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  // 0: 128-row blocks on both sides; 1: 128-row query blocks, 64-row key
+  // blocks (merged lists); 2: 64-row query blocks paired into 128-row tiles
+  const int mode = (p.block == 128 && p.block_k == 128) ? 0 : (p.block == 64 ? 2 : 1);
   CUtensorMap tm[4];
   const uint64_t inner = (uint64_t)p.H * p.d, stride = (uint64_t)p.row_stride * 2;
   const void* bases[4] = {q, k, v, dout};
-  for (int x = 0; x < 4; ++x)
-    if (!encode_tmap_2d_bf16(&tm[x], bases[x], inner, p.N, stride, 64, kTile)) return cudaErrorInvalidValue;
+  for (int x = 0; x < 4; ++x) {
+    const uint32_t box = (mode == 2 && (x == 0 || x == 3)) ? 64 : kTile;  // mode 2 loads Q, dO as 64-row boxes
+    if (!encode_tmap_2d_bf16(&tm[x], bases[x], inner, p.N, stride, 64, box)) return cudaErrorInvalidValue;
+  }
   BwdParams a{};
   a.ptr = col_ptr_t;
   a.idx = row_idx_t;
@@ -711,12 +767,11 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
   a.timeout_ns = timeout_ns;
   a.item_counter = item_counter;
   __nv_bfloat16* dqb = static_cast<__nv_bfloat16*>(dq);
-  const bool sub = p.block == 64 || p.block_k == 64;
+#define UT_BWD_LAUNCH(DD, MM) launch_bwd_fused<DD, MM>(p, tm, a, dq_acc, dqb, sms, stream)
   if (p.d == 64)
-    return sub ? launch_bwd_fused<64, true>(p, tm, a, dq_acc, dqb, sms, stream)
-               : launch_bwd_fused<64, false>(p, tm, a, dq_acc, dqb, sms, stream);
-  return sub ? launch_bwd_fused<128, true>(p, tm, a, dq_acc, dqb, sms, stream)
-             : launch_bwd_fused<128, false>(p, tm, a, dq_acc, dqb, sms, stream);
+    return mode == 0 ? UT_BWD_LAUNCH(64, 0) : (mode == 1 ? UT_BWD_LAUNCH(64, 1) : UT_BWD_LAUNCH(64, 2));
+  return mode == 0 ? UT_BWD_LAUNCH(128, 0) : (mode == 1 ? UT_BWD_LAUNCH(128, 1) : UT_BWD_LAUNCH(128, 2));
+#undef UT_BWD_LAUNCH
 }
 
 }  // namespace ut

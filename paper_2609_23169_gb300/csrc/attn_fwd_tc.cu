@@ -27,11 +27,16 @@
 // their TMA writes (128 KB), about what the two 128 x 128 x 128 products take.
 // TMEM columns: S0 [0,128), S1 [128,256), O [256,256+D), P [384,448),
 // Q [448,448+D/2).
-// Blocks of 64 rows (b_q or b_kv) are served by the same 128 x 128 tiles: an
-// item's fine key-block lists are merged into 128-row key tiles with a mask of
-// the listed 64 x 64 sub-blocks (TileList), and the softmax sets the scores of
-// unlisted sub-blocks to -inf.  Rows that see no key end with O = 0 and
-// LSE = -inf.
+// Blocks of 64 rows (b_q or b_kv) are served by the same 128 x 128 tiles:
+//   b_kv = 64:  two listed 64-row key blocks fill one 128-row key tile (two
+//               TMA boxes per operand, PairList): consecutive entries of the
+//               list for b_q = 128 (nothing discarded), the two 64-row query
+//               blocks' lists in lockstep for b_q = 64 (rows 0-63 see the low
+//               half of the tile, rows 64-127 the high half);
+//   b_q = 64, b_kv = 128:  the item's two lists are merged into 128-row key
+//               tiles with a mask of the listed 64 x 64 sub-blocks (TileList).
+// The softmax sets the scores of sub-blocks a row does not see to -inf.  Rows
+// that see no key end with O = 0 and LSE = -inf.
 // Every wait is bounded; on expiry the kernel records UT_ERR_TIMEOUT,
 // drains its own copies and MMAs, frees TMEM and returns.
 #include "common.cuh"
@@ -81,10 +86,34 @@ struct FwdParams {
   uint64_t timeout_ns;
 };
 
-template <int D, bool kSub>
+// The key steps of an item.  kMode 0: 128-row blocks on both sides (the list
+// itself); 1: 64-row query blocks, 128-row key blocks (the item's two lists
+// merged, TileList); 2: 64-row key blocks paired into 128-row tiles
+// (PairList).  next() gives the tile's key blocks (mode 2: the 64-row blocks
+// of the low and high halves, -1 if missing; otherwise lo = the 128-row key
+// tile) and the visibility bits.
+template <int kMode>
+struct KeySteps {
+  TileList<kMode == 1> tl;
+  PairList pl;
+  UT_DEV void init(const FwdParams& prm, int h, int i) {
+    if (kMode == 2) pl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile == 2);
+    else tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
+  }
+  UT_DEV int count_warp() const { return kMode == 2 ? pl.count() : tl.count_warp(); }
+  UT_DEV bool empty() const { return kMode == 2 ? pl.empty() : tl.empty(); }
+  UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
+    if (kMode == 2) return pl.next(lo, hi, bits);
+    hi = -1;
+    return tl.next(lo, bits);
+  }
+};
+
+template <int D, int kMode>
 __global__ void __launch_bounds__(kFwdThreads, 1)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                        const __grid_constant__ CUtensorMap tm_v, const FwdParams prm) {
+  constexpr bool kSub = kMode != 0;  // 64-row blocks on at least one side
   extern __shared__ uint8_t smem_raw[];
   FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   constexpr int C = FwdSmem<D>::kChunks;
@@ -147,8 +176,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int h = w / prm.nq, i = w % prm.nq;
-        TileList<kSub> tl;
-        tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
+        KeySteps<kMode> tl;
+        tl.init(prm, h, i);
         if (tl.empty()) continue;
         if (is_k) {
           if (!(ok = mbar_wait(&sm.q_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -157,15 +186,23 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
             tma_load_2d(sm.q + c * kTileChunkBytes, &tm_q, &sm.q_full, h * D + c * 64, i * kBM, pol_q);
           ++qi;
         }
-        int j;
+        int j, jh;
         uint32_t bits;
-        for (; tl.next(j, bits); ++kv) {
+        for (; tl.next(j, jh, bits); ++kv) {
           const uint32_t st = kv % kStages, n = kv / kStages;
           if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
           mbar_expect_tx(&full[st], FwdSmem<D>::kKVBytes);
-          for (int c = 0; c < C; ++c)
-            tma_load_2d(ring + st * FwdSmem<D>::kKVBytes + c * kTileChunkBytes, tmap, &full[st], h * D + c * 64,
-                        j * kBN, pol_kv);
+          uint8_t* dst = ring + st * FwdSmem<D>::kKVBytes;
+          if (kMode == 2) {  // two 64-row boxes: rows 0-63 and 64-127 of each 128-row sub-tile
+            const int b0 = PairList::load_lo(j, jh), b1 = PairList::load_hi(j, jh);
+            for (int c = 0; c < C; ++c) {
+              tma_load_2d(dst + c * kTileChunkBytes, tmap, &full[st], h * D + c * 64, b0 * 64, pol_kv);
+              tma_load_2d(dst + c * kTileChunkBytes + 64 * 128, tmap, &full[st], h * D + c * 64, b1 * 64, pol_kv);
+            }
+          } else {
+            for (int c = 0; c < C; ++c)
+              tma_load_2d(dst + c * kTileChunkBytes, tmap, &full[st], h * D + c * 64, j * kBN, pol_kv);
+          }
         }
       }
       // Drain: every copy this lane issued has landed before the CTA may exit.
@@ -186,9 +223,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       uint32_t qi = 0, oi = 0, kv0 = 0, sc0 = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-        TileList<kSub> tl;
-        tl.init(prm.row_ptr, prm.col_idx, w / prm.nq, w % prm.nq, prm.nq_fine, prm.q_rows_per_tile,
-                prm.list_shift);
+        KeySteps<kMode> tl;
+        tl.init(prm, w / prm.nq, w % prm.nq);
         const int L = tl.count_warp();
         if (L <= 0) continue;
         // Q of this item in TMEM (the softmax warps copied it there)
@@ -322,8 +358,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     };
     for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
       const int h = w / prm.nq, i = w % prm.nq;
-      TileList<kSub> tl;
-      tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
+      KeySteps<kMode> tl;
+      tl.init(prm, h, i);
       const int L = tl.count_warp();
       const int64_t grow = (int64_t)i * kBM + row;
       if (L <= 0) {
@@ -338,13 +374,13 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       if (pend && !(ok = epilogue())) break;
       pend = false;
       float m_used = 0.f, l = 0.f;
-      int j_next = 0;
+      int j_next = 0, jh_next = -1;
       uint32_t bits_next = 0;
-      tl.next(j_next, bits_next);
+      tl.next(j_next, jh_next, bits_next);
       for (int t = 0; t < L; ++t) {
-        const int j = j_next;
+        const int j = j_next, jh = jh_next;
         const uint32_t bits = bits_next;
-        if (t + 1 < L) tl.next(j_next, bits_next);  // the next tile's index, fetched a tile ahead
+        if (t + 1 < L) tl.next(j_next, jh_next, bits_next);  // the next tile's blocks, fetched a tile ahead
         const uint32_t sc = sc0 + t, sb = sc & 1, ns = sc >> 1;
         if (!(ok = warp_wait(&sm.s_full[sb], ns & 1, abort_flag, prm.status, prm.timeout_ns))) break;
         tc_fence_after();
@@ -362,12 +398,27 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         for (int x = 0; x < kBN; ++x) s[x] = __uint_as_float(r[x]);
         // ragged last key block: columns past N do not exist; 64-column
         // halves of the tile not listed for this row's half are masked
-        const int64_t nv = prm.N - (int64_t)j * kBN;
         const uint32_t cols = kSub ? (bits >> (2 * rh)) & 3u : 3u;
-        if (nv < kBN) {
+        if (kMode == 2) {  // each half holds its own 64-row key block
+          const int64_t nv0 = prm.N - 64 * (int64_t)PairList::load_lo(j, jh);
+          const int64_t nv1 = prm.N - 64 * (int64_t)PairList::load_hi(j, jh);
+          if (nv0 < 64) {
 #pragma unroll
-          for (int x = 0; x < kBN; ++x)
-            if (x >= nv) s[x] = -INFINITY;
+            for (int x = 0; x < 64; ++x)
+              if (x >= nv0) s[x] = -INFINITY;
+          }
+          if (nv1 < 64) {
+#pragma unroll
+            for (int x = 64; x < kBN; ++x)
+              if (x - 64 >= nv1) s[x] = -INFINITY;
+          }
+        } else {
+          const int64_t nv = prm.N - (int64_t)j * kBN;
+          if (nv < kBN) {
+#pragma unroll
+            for (int x = 0; x < kBN; ++x)
+              if (x >= nv) s[x] = -INFINITY;
+          }
         }
         if (kSub) {  // a masked half is the same for the whole warp (rh is per warp)
           if (!(cols & 1u)) {
@@ -464,14 +515,14 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 
 static_assert(sizeof(FwdSmem<128>) + 1024 <= 232448, "forward shared layout exceeds the per-block limit");
 
-template <int D, bool kSub>
+template <int D, int kMode>
 static cudaError_t launch_d(const AttnProblem& p, const CUtensorMap& tq, const CUtensorMap& tk,
                             const CUtensorMap& tv, const FwdParams& prm, int grid, cudaStream_t stream) {
   const size_t smem = sizeof(FwdSmem<D>) + 1024;
   cudaError_t e =
-      cudaFuncSetAttribute(attn_fwd_tc_kernel<D, kSub>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      cudaFuncSetAttribute(attn_fwd_tc_kernel<D, kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  attn_fwd_tc_kernel<D, kSub><<<grid, kFwdThreads, smem, stream>>>(tq, tk, tv, prm);
+  attn_fwd_tc_kernel<D, kMode><<<grid, kFwdThreads, smem, stream>>>(tq, tk, tv, prm);
   return cudaGetLastError();
 }
 
@@ -481,12 +532,16 @@ cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* 
   const int nt = (int)((p.N + kBM - 1) / kBM);  // 128-row tiles
   const int n_items = p.H * nt;
   if (n_items == 0) return cudaSuccess;
+  // 0: 128-row blocks on both sides; 1: 64-row query blocks, 128-row key
+  // blocks (merged lists); 2: 64-row key blocks paired into 128-row tiles
+  const int mode = (p.block == 128 && p.block_k == 128) ? 0 : (p.block_k == 64 ? 2 : 1);
   CUtensorMap tq, tk, tv;
   const uint64_t inner = (uint64_t)p.H * p.d;
   const uint64_t stride = (uint64_t)p.row_stride * 2;
+  const uint32_t kv_box = mode == 2 ? 64 : kBN;  // mode 2 loads K/V as 64-row boxes
   if (!encode_tmap_2d_bf16(&tq, q, inner, p.N, stride, 64, kBM) ||
-      !encode_tmap_2d_bf16(&tk, k, inner, p.N, stride, 64, kBN) ||
-      !encode_tmap_2d_bf16(&tv, v, inner, p.N, stride, 64, kBN))
+      !encode_tmap_2d_bf16(&tk, k, inner, p.N, stride, 64, kv_box) ||
+      !encode_tmap_2d_bf16(&tv, v, inner, p.N, stride, 64, kv_box))
     return cudaErrorInvalidValue;
   FwdParams prm{};
   prm.row_ptr = row_ptr;
@@ -505,11 +560,11 @@ cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* 
   prm.scale_log2 = p.scale * 1.4426950408889634f;
   prm.timeout_ns = timeout_ns;
   const int grid = n_items < sms ? n_items : sms;
-  const bool sub = p.block == 64 || p.block_k == 64;
+#define UT_FWD_LAUNCH(DD, MM) launch_d<DD, MM>(p, tq, tk, tv, prm, grid, stream)
   if (p.d == 64)
-    return sub ? launch_d<64, true>(p, tq, tk, tv, prm, grid, stream) : launch_d<64, false>(p, tq, tk, tv, prm, grid, stream);
-  return sub ? launch_d<128, true>(p, tq, tk, tv, prm, grid, stream)
-             : launch_d<128, false>(p, tq, tk, tv, prm, grid, stream);
+    return mode == 0 ? UT_FWD_LAUNCH(64, 0) : (mode == 1 ? UT_FWD_LAUNCH(64, 1) : UT_FWD_LAUNCH(64, 2));
+  return mode == 0 ? UT_FWD_LAUNCH(128, 0) : (mode == 1 ? UT_FWD_LAUNCH(128, 1) : UT_FWD_LAUNCH(128, 2));
+#undef UT_FWD_LAUNCH
 }
 
 }  // namespace ut

@@ -292,6 +292,69 @@ struct TileList {
   }
 };
 
+// 64-row blocks paired into 128-row tiles.  The tensor cores run 128 x 128
+// tiles at full rate (an N = 64 product costs 44 cycles against 64 for
+// N = 128, and M = 64 runs at the rate of M = 128), so a listed 64-row block
+// of the listed side is loaded as one half of a 128-row operand tile (two
+// 64-row TMA boxes) and paired with another one:
+//   one list  (the item is one block of the listing side, 128 rows): step t
+//             takes the consecutive entries (L[2t], L[2t+1]); every row of
+//             the item sees both halves (no work is discarded);
+//   two lists (the item holds two 64-row blocks a, b of the listing side):
+//             step t takes (a[t], b[t]); rows 0-63 of the item see the low
+//             half, rows 64-127 the high half.
+// A missing entry is -1: that half is masked, and the loader fills it with
+// the other half's block so that it holds finite values.
+// bits: bit (2 * r + c) = rows r * 64 .. r * 64 + 63 of the item see columns
+// c * 64 .. c * 64 + 63 of the tile (the encoding TileList uses).
+struct PairList {
+  const int32_t* a;
+  const int32_t* b;
+  int na, nb, t;
+  bool two;
+
+  // item = block t of head h on the listing side: one list (two = false) or
+  // the two 64-row blocks 2 * item and 2 * item + 1 (two = true); nfine list
+  // rows per head.
+  UT_DEV void init(const int32_t* ptr, const int32_t* idx, int h, int item, int nfine, bool item_has_two) {
+    const int64_t base = (int64_t)h * nfine;
+    two = item_has_two;
+    const int r0 = two ? 2 * item : item;
+    const int s0 = ptr[base + r0];
+    a = idx + s0;
+    na = ptr[base + r0 + 1] - s0;
+    b = a;
+    nb = 0;
+    if (two && r0 + 1 < nfine) {
+      const int s1 = ptr[base + r0 + 1];
+      b = idx + s1;
+      nb = ptr[base + r0 + 2] - s1;
+    }
+    t = 0;
+  }
+  UT_DEV int count() const { return two ? (na > nb ? na : nb) : (na + 1) / 2; }
+  UT_DEV bool empty() const { return na == 0 && nb == 0; }
+  // next pair: the 64-row blocks of the low and high halves (never both -1)
+  // and the visibility bits
+  UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
+    if (t >= count()) return false;
+    if (two) {
+      lo = t < na ? a[t] : -1;
+      hi = t < nb ? b[t] : -1;
+      bits = (lo >= 0 ? 1u : 0u) | (hi >= 0 ? 8u : 0u);
+    } else {
+      lo = a[2 * t];
+      hi = 2 * t + 1 < na ? a[2 * t + 1] : -1;
+      bits = hi >= 0 ? 15u : 5u;
+    }
+    ++t;
+    return true;
+  }
+  // the blocks the loader puts into the two halves (a missing one repeats the other)
+  UT_DEV static int load_lo(int lo, int hi) { return lo >= 0 ? lo : hi; }
+  UT_DEV static int load_hi(int lo, int hi) { return hi >= 0 ? hi : lo; }
+};
+
 // ---------------------------------------------------------------- tcgen05
 UT_DEV void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
