@@ -169,21 +169,32 @@ UT_DEV void red_add_f32(float* p, float v) {
 
 // The query steps of an item.  kMode 0: 128-row blocks on both sides; 1:
 // 128-row query blocks, 64-row key blocks (merged lists, TileList); 2: 64-row
-// query blocks paired into 128-row tiles (PairList).  next() gives the tile's
-// query blocks (mode 2: the 64-row blocks of the low and high halves, -1 if
-// missing; otherwise lo = the 128-row query tile) and the visibility bits.
+// query blocks paired into 128-row tiles (PairList, one list); 3: 64-row
+// blocks on both sides, per item whichever of the merged tiles and the paired
+// lists takes fewer steps.  next() gives the tile's query blocks (paired: the
+// 64-row blocks of the low and high halves, -1 if missing; merged: lo = the
+// 128-row query tile) and the visibility bits.  In mode 3 init() takes the
+// item's choice from the lists' first and last entries (pairing_is_shorter),
+// the same in every role.
 template <int kMode>
 struct QuerySteps {
-  TileList<kMode == 1> tl;
+  TileList<kMode == 1 || kMode == 3> tl;
   PairList pl;
+  bool pair;
   UT_DEV void init(const BwdParams& prm, int h, int j) {
+    if (kMode != 2) tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
     if (kMode == 2) pl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile == 2);
-    else tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
+    pair = kMode == 2;
+    if constexpr (kMode == 3) pair = pairing_is_shorter(tl);
   }
-  UT_DEV int count_warp() const { return kMode == 2 ? pl.count() : tl.count_warp(); }
+  UT_DEV int count_warp() const {
+    if (kMode == 3 && pair) return tl.na > tl.nb ? tl.na : tl.nb;
+    return kMode == 2 ? pl.count() : tl.count_warp();
+  }
   UT_DEV bool empty() const { return kMode == 2 ? pl.empty() : tl.empty(); }
   UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
     if (kMode == 2) return pl.next(lo, hi, bits);
+    if (kMode == 3 && pair) return PairList::step_two(tl.a, tl.b, tl.na, tl.nb, tl.pa, lo, hi, bits);
     hi = -1;
     return tl.next(lo, bits);
   }
@@ -193,6 +204,7 @@ template <int D, int kMode>
 __global__ void __launch_bounds__(kFuThreads, 1)
     bwd_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                      const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+                     const __grid_constant__ CUtensorMap tm_q64, const __grid_constant__ CUtensorMap tm_do64,
                      const BwdParams prm, float* __restrict__ dq_acc) {
   constexpr bool kSub = kMode != 0;  // 64-row blocks on at least one side
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -279,14 +291,17 @@ __global__ void __launch_bounds__(kFuThreads, 1)
           tma_prefetch_desc(&tm_q);
           tma_prefetch_desc(&tm_k);
           tma_prefetch_desc(&tm_v);
+          if (kMode >= 2) tma_prefetch_desc(&tm_q64);
         } else {
           tma_prefetch_desc(&tm_do);
+          if (kMode >= 2) tma_prefetch_desc(&tm_do64);
         }
         const uint64_t pol_qd = policy_evict_last(), pol_kv = policy_evict_first();
         uint64_t* full = is_q ? sm.q_full : sm.do_full;
         uint64_t* empty = is_q ? sm.q_empty : sm.do_empty;
         uint8_t* ring = is_q ? &sm.q[0][0] : &sm.dout[0][0];
         const void* tmap = is_q ? static_cast<const void*>(&tm_q) : static_cast<const void*>(&tm_do);
+        const void* tmap64 = is_q ? static_cast<const void*>(&tm_q64) : static_cast<const void*>(&tm_do64);
         const uint32_t nst = is_q ? kFuQStages : kFuDoStages;
         uint32_t ki = 0, qd = 0, kk = 0;
         bool ok = true;
@@ -324,11 +339,11 @@ __global__ void __launch_bounds__(kFuThreads, 1)
             if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
             mbar_expect_tx(&full[st], TB);
             uint8_t* dst = ring + st * TB;
-            if (kMode == 2) {  // two 64-row boxes: rows 0-63 and 64-127 of each 128-row sub-tile
+            if (tl.pair) {  // two 64-row boxes: rows 0-63 and 64-127 of each 128-row sub-tile
               const int b0 = PairList::load_lo(i, ih), b1 = PairList::load_hi(i, ih);
               for (int c = 0; c < C; ++c) {
-                tma_load_2d(dst + c * kChunk, tmap, &full[st], h * D + c * 64, b0 * 64, pol_qd);
-                tma_load_2d(dst + c * kChunk + 64 * 128, tmap, &full[st], h * D + c * 64, b1 * 64, pol_qd);
+                tma_load_2d(dst + c * kChunk, tmap64, &full[st], h * D + c * 64, b0 * 64, pol_qd);
+                tma_load_2d(dst + c * kChunk + 64 * 128, tmap64, &full[st], h * D + c * 64, b1 * 64, pol_qd);
               }
             } else {
               for (int c = 0; c < C; ++c)
@@ -480,7 +495,7 @@ __global__ void __launch_bounds__(kFuThreads, 1)
       const uint32_t qcol = tid & (kTile - 1), qhalf = qcol >> 6;
       const float* rv_src = (tid < kTile ? prm.lse2 : prm.dsum) + (int64_t)h * prm.Np + (qcol & 63);
       auto rv_row = [&](int lo, int hi) -> int64_t {  // first row of this thread's 64-row query half
-        if (kMode == 2) return 64 * (int64_t)(qhalf ? PairList::load_hi(lo, hi) : PairList::load_lo(lo, hi));
+        if (tl.pair) return 64 * (int64_t)(qhalf ? PairList::load_hi(lo, hi) : PairList::load_lo(lo, hi));
         return (int64_t)lo * kTile + 64 * qhalf;
       };
       int i_next, ih_next;
@@ -632,11 +647,11 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         tc_fence_after();
 #pragma unroll
         for (int g = 0; g < 2; ++g) {
-          // query half g of the tile: rows of 64-row block lo / hi (mode 2), or
+          // query half g of the tile: rows of 64-row block lo / hi (paired), or
           // rows g * 64 .. of the 128-row query block; a missing block (-1)
           // has dS^T = 0 there and is not added
-          const int blk = kMode == 2 ? (g ? ih : i) : 0;
-          const int64_t row0 = kMode == 2 ? 64 * (int64_t)blk : (int64_t)i * kTile + 64 * g;
+          const int blk = tl.pair ? (g ? ih : i) : 0;
+          const int64_t row0 = tl.pair ? 64 * (int64_t)blk : (int64_t)i * kTile + 64 * g;
           float* dst = dq_acc + (((int64_t)h * prm.Np + row0) * D + dcol);
           uint32_t r[64];
           tmem_ld64(tmem + lane_base + kColRQ + g * 64, r);
@@ -705,7 +720,7 @@ static cudaError_t launch_bwd_fused(const AttnProblem& p, const CUtensorMap* tm,
   e = cudaFuncGetAttributes(&fa, bwd_fused_kernel<D, kMode>);
   if (e != cudaSuccess) return e;
   if (fa.numRegs != kFuRegLaunch) return cudaErrorInvalidConfiguration;
-  bwd_fused_kernel<D, kMode><<<grid, kFuThreads, smem, s>>>(tm[0], tm[1], tm[2], tm[3], prm, dq_acc);
+  bwd_fused_kernel<D, kMode><<<grid, kFuThreads, smem, s>>>(tm[0], tm[1], tm[2], tm[3], tm[4], tm[5], prm, dq_acc);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int64_t n8 = p.N * p.H * D / 8;
@@ -736,15 +751,15 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   // 0: 128-row blocks on both sides; 1: 128-row query blocks, 64-row key
-  // blocks (merged lists); 2: 64-row query blocks paired into 128-row tiles
-  const int mode = (p.block == 128 && p.block_k == 128) ? 0 : (p.block == 64 ? 2 : 1);
-  CUtensorMap tm[4];
+  // blocks (merged lists); 2: 64-row query blocks, 128-row key blocks, paired
+  // into 128-row tiles; 3: 64-row blocks on both sides, merged or paired per item
+  const int mode = p.block == 128 ? (p.block_k == 128 ? 0 : 1) : (p.block_k == 128 ? 2 : 3);
+  CUtensorMap tm[6];  // Q, K, V, dO as 128-row boxes, then Q and dO as 64-row boxes
   const uint64_t inner = (uint64_t)p.H * p.d, stride = (uint64_t)p.row_stride * 2;
-  const void* bases[4] = {q, k, v, dout};
-  for (int x = 0; x < 4; ++x) {
-    const uint32_t box = (mode == 2 && (x == 0 || x == 3)) ? 64 : kTile;  // mode 2 loads Q, dO as 64-row boxes
-    if (!encode_tmap_2d_bf16(&tm[x], bases[x], inner, p.N, stride, 64, box)) return cudaErrorInvalidValue;
-  }
+  const void* bases[6] = {q, k, v, dout, q, dout};
+  for (int x = 0; x < 6; ++x)
+    if (!encode_tmap_2d_bf16(&tm[x], bases[x], inner, p.N, stride, 64, x < 4 ? kTile : 64))
+      return cudaErrorInvalidValue;
   BwdParams a{};
   a.ptr = col_ptr_t;
   a.idx = row_idx_t;
@@ -768,9 +783,12 @@ cudaError_t launch_attn_bwd_tc(const AttnProblem& p, const void* q, const void* 
   a.item_counter = item_counter;
   __nv_bfloat16* dqb = static_cast<__nv_bfloat16*>(dq);
 #define UT_BWD_LAUNCH(DD, MM) launch_bwd_fused<DD, MM>(p, tm, a, dq_acc, dqb, sms, stream)
-  if (p.d == 64)
-    return mode == 0 ? UT_BWD_LAUNCH(64, 0) : (mode == 1 ? UT_BWD_LAUNCH(64, 1) : UT_BWD_LAUNCH(64, 2));
-  return mode == 0 ? UT_BWD_LAUNCH(128, 0) : (mode == 1 ? UT_BWD_LAUNCH(128, 1) : UT_BWD_LAUNCH(128, 2));
+#define UT_BWD_MODES(DD)                                                                    \
+  (mode == 0 ? UT_BWD_LAUNCH(DD, 0)                                                         \
+             : (mode == 1 ? UT_BWD_LAUNCH(DD, 1) : (mode == 2 ? UT_BWD_LAUNCH(DD, 2) : UT_BWD_LAUNCH(DD, 3))))
+  if (p.d == 64) return UT_BWD_MODES(64);
+  return UT_BWD_MODES(128);
+#undef UT_BWD_MODES
 #undef UT_BWD_LAUNCH
 }
 

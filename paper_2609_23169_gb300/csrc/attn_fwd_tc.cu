@@ -89,21 +89,33 @@ struct FwdParams {
 // The key steps of an item.  kMode 0: 128-row blocks on both sides (the list
 // itself); 1: 64-row query blocks, 128-row key blocks (the item's two lists
 // merged, TileList); 2: 64-row key blocks paired into 128-row tiles
-// (PairList).  next() gives the tile's key blocks (mode 2: the 64-row blocks
-// of the low and high halves, -1 if missing; otherwise lo = the 128-row key
-// tile) and the visibility bits.
+// (PairList); 3: 64-row blocks on both sides, per item whichever of the
+// merged tiles and the paired lists takes fewer steps (pairing discards half
+// of each tile but merging discards the unlisted sub-blocks, most of them
+// when the lists are sparse; dense or clustered lists merge into fewer
+// tiles).  next() gives the tile's key blocks (paired: the 64-row blocks of
+// the low and high halves, -1 if missing; merged: lo = the 128-row key tile)
+// and the visibility bits.  In mode 3 init() takes the item's choice from the
+// lists' first and last entries (pairing_is_shorter), the same in every role.
 template <int kMode>
 struct KeySteps {
-  TileList<kMode == 1> tl;
+  TileList<kMode == 1 || kMode == 3> tl;
   PairList pl;
+  bool pair;
   UT_DEV void init(const FwdParams& prm, int h, int i) {
+    if (kMode != 2) tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
     if (kMode == 2) pl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile == 2);
-    else tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
+    pair = kMode == 2;
+    if constexpr (kMode == 3) pair = pairing_is_shorter(tl);
   }
-  UT_DEV int count_warp() const { return kMode == 2 ? pl.count() : tl.count_warp(); }
+  UT_DEV int count_warp() const {
+    if (kMode == 3 && pair) return tl.na > tl.nb ? tl.na : tl.nb;
+    return kMode == 2 ? pl.count() : tl.count_warp();
+  }
   UT_DEV bool empty() const { return kMode == 2 ? pl.empty() : tl.empty(); }
   UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
     if (kMode == 2) return pl.next(lo, hi, bits);
+    if (kMode == 3 && pair) return PairList::step_two(tl.a, tl.b, tl.na, tl.nb, tl.pa, lo, hi, bits);
     hi = -1;
     return tl.next(lo, bits);
   }
@@ -112,7 +124,8 @@ struct KeySteps {
 template <int D, int kMode>
 __global__ void __launch_bounds__(kFwdThreads, 1)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                       const __grid_constant__ CUtensorMap tm_v, const FwdParams prm) {
+                       const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_k64,
+                       const __grid_constant__ CUtensorMap tm_v64, const FwdParams prm) {
   constexpr bool kSub = kMode != 0;  // 64-row blocks on at least one side
   extern __shared__ uint8_t smem_raw[];
   FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -163,8 +176,10 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       if (is_k) {
         tma_prefetch_desc(&tm_q);
         tma_prefetch_desc(&tm_k);
+        if (kMode >= 2) tma_prefetch_desc(&tm_k64);
       } else {
         tma_prefetch_desc(&tm_v);
+        if (kMode >= 2) tma_prefetch_desc(&tm_v64);
       }
       const uint64_t pol_kv = policy_evict_last();
       const uint64_t pol_q = policy_evict_first();
@@ -172,6 +187,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       uint64_t* empty = is_k ? sm.k_empty : sm.v_empty;
       uint8_t* ring = is_k ? &sm.k[0][0] : &sm.v[0][0];
       const void* tmap = is_k ? static_cast<const void*>(&tm_k) : static_cast<const void*>(&tm_v);
+      const void* tmap64 = is_k ? static_cast<const void*>(&tm_k64) : static_cast<const void*>(&tm_v64);
       uint32_t qi = 0, kv = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
@@ -193,11 +209,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           if (!(ok = mbar_wait(&empty[st], (n & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
           mbar_expect_tx(&full[st], FwdSmem<D>::kKVBytes);
           uint8_t* dst = ring + st * FwdSmem<D>::kKVBytes;
-          if (kMode == 2) {  // two 64-row boxes: rows 0-63 and 64-127 of each 128-row sub-tile
+          if (tl.pair) {  // two 64-row boxes: rows 0-63 and 64-127 of each 128-row sub-tile
             const int b0 = PairList::load_lo(j, jh), b1 = PairList::load_hi(j, jh);
             for (int c = 0; c < C; ++c) {
-              tma_load_2d(dst + c * kTileChunkBytes, tmap, &full[st], h * D + c * 64, b0 * 64, pol_kv);
-              tma_load_2d(dst + c * kTileChunkBytes + 64 * 128, tmap, &full[st], h * D + c * 64, b1 * 64, pol_kv);
+              tma_load_2d(dst + c * kTileChunkBytes, tmap64, &full[st], h * D + c * 64, b0 * 64, pol_kv);
+              tma_load_2d(dst + c * kTileChunkBytes + 64 * 128, tmap64, &full[st], h * D + c * 64, b1 * 64, pol_kv);
             }
           } else {
             for (int c = 0; c < C; ++c)
@@ -399,7 +415,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         // ragged last key block: columns past N do not exist; 64-column
         // halves of the tile not listed for this row's half are masked
         const uint32_t cols = kSub ? (bits >> (2 * rh)) & 3u : 3u;
-        if (kMode == 2) {  // each half holds its own 64-row key block
+        if (tl.pair) {  // each half holds its own 64-row key block
           const int64_t nv0 = prm.N - 64 * (int64_t)PairList::load_lo(j, jh);
           const int64_t nv1 = prm.N - 64 * (int64_t)PairList::load_hi(j, jh);
           if (nv0 < 64) {
@@ -517,12 +533,13 @@ static_assert(sizeof(FwdSmem<128>) + 1024 <= 232448, "forward shared layout exce
 
 template <int D, int kMode>
 static cudaError_t launch_d(const AttnProblem& p, const CUtensorMap& tq, const CUtensorMap& tk,
-                            const CUtensorMap& tv, const FwdParams& prm, int grid, cudaStream_t stream) {
+                            const CUtensorMap& tv, const CUtensorMap& tk64, const CUtensorMap& tv64,
+                            const FwdParams& prm, int grid, cudaStream_t stream) {
   const size_t smem = sizeof(FwdSmem<D>) + 1024;
   cudaError_t e =
       cudaFuncSetAttribute(attn_fwd_tc_kernel<D, kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  attn_fwd_tc_kernel<D, kMode><<<grid, kFwdThreads, smem, stream>>>(tq, tk, tv, prm);
+  attn_fwd_tc_kernel<D, kMode><<<grid, kFwdThreads, smem, stream>>>(tq, tk, tv, tk64, tv64, prm);
   return cudaGetLastError();
 }
 
@@ -533,15 +550,17 @@ cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* 
   const int n_items = p.H * nt;
   if (n_items == 0) return cudaSuccess;
   // 0: 128-row blocks on both sides; 1: 64-row query blocks, 128-row key
-  // blocks (merged lists); 2: 64-row key blocks paired into 128-row tiles
-  const int mode = (p.block == 128 && p.block_k == 128) ? 0 : (p.block_k == 64 ? 2 : 1);
-  CUtensorMap tq, tk, tv;
+  // blocks (merged lists); 2: 128-row query blocks, 64-row key blocks paired
+  // into 128-row tiles; 3: 64-row blocks on both sides, merged or paired per item
+  const int mode = p.block == 128 ? (p.block_k == 128 ? 0 : 2) : (p.block_k == 128 ? 1 : 3);
+  CUtensorMap tq, tk, tv, tk64, tv64;  // K / V as 128-row and as 64-row boxes
   const uint64_t inner = (uint64_t)p.H * p.d;
   const uint64_t stride = (uint64_t)p.row_stride * 2;
-  const uint32_t kv_box = mode == 2 ? 64 : kBN;  // mode 2 loads K/V as 64-row boxes
   if (!encode_tmap_2d_bf16(&tq, q, inner, p.N, stride, 64, kBM) ||
-      !encode_tmap_2d_bf16(&tk, k, inner, p.N, stride, 64, kv_box) ||
-      !encode_tmap_2d_bf16(&tv, v, inner, p.N, stride, 64, kv_box))
+      !encode_tmap_2d_bf16(&tk, k, inner, p.N, stride, 64, kBN) ||
+      !encode_tmap_2d_bf16(&tv, v, inner, p.N, stride, 64, kBN) ||
+      !encode_tmap_2d_bf16(&tk64, k, inner, p.N, stride, 64, 64) ||
+      !encode_tmap_2d_bf16(&tv64, v, inner, p.N, stride, 64, 64))
     return cudaErrorInvalidValue;
   FwdParams prm{};
   prm.row_ptr = row_ptr;
@@ -560,10 +579,13 @@ cudaError_t launch_attn_fwd_tc(const AttnProblem& p, const void* q, const void* 
   prm.scale_log2 = p.scale * 1.4426950408889634f;
   prm.timeout_ns = timeout_ns;
   const int grid = n_items < sms ? n_items : sms;
-#define UT_FWD_LAUNCH(DD, MM) launch_d<DD, MM>(p, tq, tk, tv, prm, grid, stream)
-  if (p.d == 64)
-    return mode == 0 ? UT_FWD_LAUNCH(64, 0) : (mode == 1 ? UT_FWD_LAUNCH(64, 1) : UT_FWD_LAUNCH(64, 2));
-  return mode == 0 ? UT_FWD_LAUNCH(128, 0) : (mode == 1 ? UT_FWD_LAUNCH(128, 1) : UT_FWD_LAUNCH(128, 2));
+#define UT_FWD_LAUNCH(DD, MM) launch_d<DD, MM>(p, tq, tk, tv, tk64, tv64, prm, grid, stream)
+#define UT_FWD_MODES(DD)                                                                    \
+  (mode == 0 ? UT_FWD_LAUNCH(DD, 0)                                                         \
+             : (mode == 1 ? UT_FWD_LAUNCH(DD, 1) : (mode == 2 ? UT_FWD_LAUNCH(DD, 2) : UT_FWD_LAUNCH(DD, 3))))
+  if (p.d == 64) return UT_FWD_MODES(64);
+  return UT_FWD_MODES(128);
+#undef UT_FWD_MODES
 #undef UT_FWD_LAUNCH
 }
 

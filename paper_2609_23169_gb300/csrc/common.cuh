@@ -336,13 +336,20 @@ struct PairList {
   UT_DEV bool empty() const { return na == 0 && nb == 0; }
   // next pair: the 64-row blocks of the low and high halves (never both -1)
   // and the visibility bits
+  // step t of two lists in lockstep (also used on a TileList's own lists)
+  UT_DEV static bool step_two(const int32_t* a, const int32_t* b, int na, int nb, int& t, int& lo, int& hi,
+                              uint32_t& bits) {
+    if (t >= (na > nb ? na : nb)) return false;
+    lo = t < na ? a[t] : -1;
+    hi = t < nb ? b[t] : -1;
+    bits = (lo >= 0 ? 1u : 0u) | (hi >= 0 ? 8u : 0u);
+    ++t;
+    return true;
+  }
   UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
+    if (two) return step_two(a, b, na, nb, t, lo, hi, bits);
     if (t >= count()) return false;
-    if (two) {
-      lo = t < na ? a[t] : -1;
-      hi = t < nb ? b[t] : -1;
-      bits = (lo >= 0 ? 1u : 0u) | (hi >= 0 ? 8u : 0u);
-    } else {
+    {
       lo = a[2 * t];
       hi = 2 * t + 1 < na ? a[2 * t + 1] : -1;
       bits = hi >= 0 ? 15u : 5u;
@@ -354,6 +361,32 @@ struct PairList {
   UT_DEV static int load_lo(int lo, int hi) { return lo >= 0 ? lo : hi; }
   UT_DEV static int load_hi(int lo, int hi) { return hi >= 0 ? hi : lo; }
 };
+
+// With 64-row blocks on both sides an item can merge its two lists into
+// 128-row tiles (TileList) or step through them in lockstep (the two-list
+// form of PairList, run on the TileList's own lists); each step costs one
+// 128 x 128 tile.  Pairing takes max(na, nb) steps.  Merging takes the number
+// of distinct tiles, at most the entry count and at most the tiles spanned
+// between the first and the last entry: few for dense or clustered lists,
+// about na + nb for sparse scattered ones.  Pairing is chosen when it takes
+// fewer steps than that bound.  Only the lists' first and last entries are
+// read, so every role takes the same choice at the cost of four loads.
+UT_DEV bool pairing_is_shorter(const TileList<true>& tl) {
+  if (tl.na + tl.nb == 0) return false;
+  int first = 0x7fffffff, last = -1;
+  if (tl.na > 0) {
+    first = tl.a[0];
+    last = tl.a[tl.na - 1];
+  }
+  if (tl.nb > 0) {
+    first = tl.b[0] < first ? tl.b[0] : first;
+    last = tl.b[tl.nb - 1] > last ? tl.b[tl.nb - 1] : last;
+  }
+  const int spanned = (last >> tl.shift) - (first >> tl.shift) + 1;
+  const int entries = tl.na + tl.nb;
+  const int paired = tl.na > tl.nb ? tl.na : tl.nb;
+  return paired < (spanned < entries ? spanned : entries);
+}
 
 // ---------------------------------------------------------------- tcgen05
 UT_DEV void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
