@@ -614,14 +614,17 @@ def time_sampler_steps(w, dev, hbm_peak: float, reps: int = 20) -> dict:
             tot += e0.elapsed_time(e1)
         return tot / reps
 
+    zc = torch.empty_like(v)
     ms_e = timed(lambda: u.ut_fg_euler_update(idx, n, z, v, x["dt"], status=st))
+    ms_g = timed(lambda: u.ut_fg_euler_update_gather(idx, n, z, v, x["dt"], zc=zc, status=st))
     ms_c = timed(lambda: u.ut_fg_composite(mask, z, tile))
     u.check_status(st)
     b_e = n * (4 + 3 * row)            # idx, v read, z read + write (foreground rows)
+    b_g = n * (4 + 4 * row)            # the same and the compacted rows written for the next step
     b_c = T + (T - n) * row            # mask read, background rows written
     out = {"workload": f"{w.name} target canvas: {T} tokens, {n} foreground, 64 channels bf16, "
                        f"tile of {x['period']} rows", "l2": "flushed before each call by reading 256 MB"}
-    for name, ms, b in (("euler_update", ms_e, b_e), ("composite", ms_c, b_c)):
+    for name, ms, b in (("euler_update", ms_e, b_e), ("euler_update_gather", ms_g, b_g), ("composite", ms_c, b_c)):
         gbs = b / (ms * 1e-3) / 1e9
         out[name] = {"ms": round(ms, 5), "bytes": int(b), "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4)}
     return out

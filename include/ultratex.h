@@ -236,6 +236,19 @@ ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void*
                              int32_t channels, int32_t dtype, float dt, int32_t* dev_status,
                              void* stream);
 
+/* The sparse Euler step fused with the gather of the next denoising step:
+ * the update of ut_fg_euler_update, and the updated row also written to
+ *   zc[n] = z[idx[n]] (after the update)  for n < n,
+ * the compacted latent that the next step's model call takes (Sec. 3.2: the
+ * model runs on the retained tokens only, gathered by M_fg every step).  One
+ * pass reads idx, v and z's retained rows once and writes them to z and zc.
+ *   zc  [n, channels] device (dtype), 16-byte aligned; may not overlap z or v.
+ * Other arguments, rounding and errors as ut_fg_euler_update (rows whose idx
+ * is outside [0, T) are skipped in both outputs). */
+ut_status ut_fg_euler_update_gather(const int32_t* idx, int64_t n, void* z, const void* v, void* zc, int64_t T,
+                                    int32_t channels, int32_t dtype, float dt, int32_t* dev_status,
+                                    void* stream);
+
 /* ------------------------------------------------------------------------
  * Composite latent for decoding (Sec. 3.4, Eq. mixed_latent):
  *   z[t] = z_bg[t mod period]  where mask[t] == 0;  foreground rows unchanged.

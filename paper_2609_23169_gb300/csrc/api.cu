@@ -238,8 +238,8 @@ int32_t ut_device_accessible(const void* ptr) {
   return a.type == cudaMemoryTypeHost && a.devicePointer == ptr ? 1 : 0;
 }
 
-ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int32_t channels,
-                             int32_t dtype, float dt, int32_t* dev_status, void* stream) {
+static ut_status euler_checked(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int32_t channels,
+                               int32_t dtype, float dt, int32_t* dev_status, void* zc, bool with_zc, void* stream) {
   if (n < 0 || T < 0 || n > T || channels <= 0) return UT_ERR_INVALID_ARG;
   if (dtype != UT_BF16 && dtype != UT_F32) return UT_ERR_INVALID_ARG;
   const int64_t row_bytes = (int64_t)channels * (dtype == UT_BF16 ? 2 : 4);
@@ -247,8 +247,20 @@ ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void*
   if (!isfinite(dt)) return UT_ERR_INVALID_ARG;
   if (n == 0) return UT_OK;
   if (!idx || !z || !v || !aligned16(z) || !aligned16(v)) return UT_ERR_INVALID_ARG;
+  if (with_zc && (!zc || !aligned16(zc))) return UT_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  return from_cuda(launch_fg_euler(idx, n, z, v, T, row_bytes, dtype == UT_BF16, dt, dev_status, device_sms(), s));
+  return from_cuda(launch_fg_euler(idx, n, z, v, T, row_bytes, dtype == UT_BF16, dt, dev_status, with_zc ? zc : nullptr,
+                                   device_sms(), s));
+}
+
+ut_status ut_fg_euler_update(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int32_t channels,
+                             int32_t dtype, float dt, int32_t* dev_status, void* stream) {
+  return euler_checked(idx, n, z, v, T, channels, dtype, dt, dev_status, nullptr, false, stream);
+}
+
+ut_status ut_fg_euler_update_gather(const int32_t* idx, int64_t n, void* z, const void* v, void* zc, int64_t T,
+                                    int32_t channels, int32_t dtype, float dt, int32_t* dev_status, void* stream) {
+  return euler_checked(idx, n, z, v, T, channels, dtype, dt, dev_status, zc, true, stream);
 }
 
 ut_status ut_fg_composite(const uint8_t* mask, int64_t T, void* z, const void* z_bg, int64_t period,

@@ -18,7 +18,7 @@ cudaError_t launch_fg_scatter(const int32_t* idx, int64_t N, int n_tensors, cons
 
 // sampler.cu
 cudaError_t launch_fg_euler(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int64_t row_bytes,
-                            bool bf16, float dt, int32_t* status, int sms, cudaStream_t stream);
+                            bool bf16, float dt, int32_t* status, void* zc, int sms, cudaStream_t stream);
 cudaError_t launch_fg_composite(const uint8_t* mask, int64_t T, void* z, const void* tile, int64_t period,
                                 int64_t row_bytes, int sms, cudaStream_t stream);
 

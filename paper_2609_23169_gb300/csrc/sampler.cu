@@ -4,7 +4,11 @@
 //                        z[idx[n]] += dt * v[n], dt = t_prev - t_curr; the
 //                        background rows are not touched.  One fused
 //                        multiply-add in fp32 per element, rounded once to the
-//                        storage type (bf16 or fp32).
+//                        storage type (bf16 or fp32).  Optionally the updated
+//                        row is also written to zc[n]: the compacted latent
+//                        the next denoising step feeds the model (the gather
+//                        of Background Token Dropping fused with the update,
+//                        so that step reads z's foreground rows once).
 //   fg_composite_kernel  composite latent for decoding (Sec. 3.4,
 //                        Eq. mixed_latent): background row t of z takes row
 //                        t mod P of the canonical background tile; foreground
@@ -35,15 +39,17 @@ UT_DEV uint32_t euler_bf16x2(uint32_t z, uint32_t v, float dt) {
   return pack_bf16x2(fmaf(dt, bf16_lo(v), bf16_lo(z)), fmaf(dt, bf16_hi(v), bf16_hi(z)));
 }
 
-template <bool kBf16>
+template <bool kBf16, typename I>
 __global__ void __launch_bounds__(kSamplerThreads) fg_euler_kernel(const int32_t* __restrict__ idx, int64_t n,
                                                                    uint8_t* __restrict__ z,
                                                                    const uint8_t* __restrict__ v, int64_t T,
-                                                                   int64_t row_bytes, float dt, int32_t* status) {
-  const int64_t V = row_bytes >> 4;
-  const int64_t total = n * V;
-  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = g / V, c = g - r * V;
+                                                                   int64_t row_bytes, float dt, int32_t* status,
+                                                                   uint8_t* __restrict__ zc) {
+  // I: the index type of the vector count (32-bit division when it fits)
+  const I V = (I)(row_bytes >> 4);
+  const I total = (I)n * V;
+  for (I g = (I)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (I)gridDim.x * blockDim.x) {
+    const I r = g / V, c = g - r * V;
     const int64_t t = idx[r];
     if (t < 0 || t >= T) {  // an index outside the canvas: skip the row, report it
       if (c == 0) set_status(status, UT_ERR_INVALID_ARG);
@@ -64,6 +70,7 @@ __global__ void __launch_bounds__(kSamplerThreads) fg_euler_kernel(const int32_t
       zz.w = __float_as_uint(fmaf(dt, __uint_as_float(vv.w), __uint_as_float(zz.w)));
     }
     st_v4(zp, zz);
+    if (zc) st_v4(zc + (int64_t)r * row_bytes + ((int64_t)c << 4), zz);
   }
 }
 
@@ -82,17 +89,26 @@ __global__ void __launch_bounds__(kSamplerThreads) fg_composite_kernel(const uin
 }
 
 cudaError_t launch_fg_euler(const int32_t* idx, int64_t n, void* z, const void* v, int64_t T, int64_t row_bytes,
-                            bool bf16, float dt, int32_t* status, int sms, cudaStream_t stream) {
+                            bool bf16, float dt, int32_t* status, void* zc, int sms, cudaStream_t stream) {
   if (n == 0) return cudaSuccess;
-  const int grid = stream_grid(n * (row_bytes >> 4), sms);
-  if (bf16)
-    fg_euler_kernel<true><<<grid, kSamplerThreads, 0, stream>>>(idx, n, static_cast<uint8_t*>(z),
-                                                                 static_cast<const uint8_t*>(v), T, row_bytes, dt,
-                                                                 status);
-  else
-    fg_euler_kernel<false><<<grid, kSamplerThreads, 0, stream>>>(idx, n, static_cast<uint8_t*>(z),
-                                                                  static_cast<const uint8_t*>(v), T, row_bytes, dt,
-                                                                  status);
+  const int64_t vectors = n * (row_bytes >> 4);
+  const int grid = stream_grid(vectors, sms);
+  uint8_t* zb = static_cast<uint8_t*>(z);
+  const uint8_t* vb = static_cast<const uint8_t*>(v);
+  uint8_t* zcb = static_cast<uint8_t*>(zc);
+  // the grid-stride index stays below vectors + grid * threads
+  const bool small = vectors + (int64_t)grid * kSamplerThreads < ((int64_t)1 << 31);
+  if (bf16) {
+    if (small)
+      fg_euler_kernel<true, int32_t><<<grid, kSamplerThreads, 0, stream>>>(idx, n, zb, vb, T, row_bytes, dt, status, zcb);
+    else
+      fg_euler_kernel<true, int64_t><<<grid, kSamplerThreads, 0, stream>>>(idx, n, zb, vb, T, row_bytes, dt, status, zcb);
+  } else {
+    if (small)
+      fg_euler_kernel<false, int32_t><<<grid, kSamplerThreads, 0, stream>>>(idx, n, zb, vb, T, row_bytes, dt, status, zcb);
+    else
+      fg_euler_kernel<false, int64_t><<<grid, kSamplerThreads, 0, stream>>>(idx, n, zb, vb, T, row_bytes, dt, status, zcb);
+  }
   return cudaGetLastError();
 }
 

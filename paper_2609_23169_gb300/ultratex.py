@@ -24,7 +24,7 @@ UT_MASK_TOPK, UT_MASK_BITMAP = 0, 1
 EXPORTS = (
     "ut_strerror", "ut_topk_count", "ut_fg_compact_workspace_size", "ut_fg_compact", "ut_fg_scatter",
     "ut_block_mask_workspace_size", "ut_block_mask", "ut_bsattn_fwd", "ut_bsattn_bwd_workspace_size",
-    "ut_bsattn_bwd", "ut_fg_compact_noalloc", "ut_fg_euler_update", "ut_fg_composite",
+    "ut_bsattn_bwd", "ut_fg_compact_noalloc", "ut_fg_euler_update", "ut_fg_euler_update_gather", "ut_fg_composite",
     "ut_fg_gather_rope", "ut_fg_scatter_rope", "ut_fg_mask_from_alpha", "ut_device_accessible",
 )
 
@@ -89,6 +89,8 @@ def lib() -> ctypes.CDLL:
                                 _vp, _vp, _vp, _vp, _sz, _vp, _vp]
     L.ut_fg_euler_update.restype = _i32
     L.ut_fg_euler_update.argtypes = [_vp, _i64, _vp, _vp, _i64, _i32, _i32, _flt, _vp, _vp]
+    L.ut_fg_euler_update_gather.restype = _i32
+    L.ut_fg_euler_update_gather.argtypes = [_vp, _i64, _vp, _vp, _vp, _i64, _i32, _i32, _flt, _vp, _vp]
     L.ut_fg_composite.restype = _i32
     L.ut_fg_composite.argtypes = [_vp, _i64, _vp, _vp, _i64, _i64, _vp]
     L.ut_fg_gather_rope.restype = _i32
@@ -295,6 +297,29 @@ def ut_fg_euler_update(idx: torch.Tensor, n: int, z: torch.Tensor, v: torch.Tens
     dtype = UT_BF16 if z.dtype == torch.bfloat16 else UT_F32
     st = lib().ut_fg_euler_update(_p(idx), int(n), _p(z), _p(v), T, C, dtype, float(dt), _p(status), _stream())
     _check("ut_fg_euler_update", st)
+
+
+def ut_fg_euler_update_gather(idx: torch.Tensor, n: int, z: torch.Tensor, v: torch.Tensor, dt: float,
+                              zc: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Sparse Euler step in place and the gather of the updated rows:
+    z[idx[i]] += dt * v[i]; zc[i] = z[idx[i]] for i < n.  Returns zc."""
+    if z.dtype not in (torch.bfloat16, torch.float32) or v.dtype != z.dtype:
+        raise ValueError("z and v must share dtype bf16 or fp32")
+    if not (z.is_contiguous() and v.is_contiguous()):
+        raise ValueError("z and v must be contiguous")
+    T = z.shape[0]
+    C = z[0].numel() if T > 0 else (v[0].numel() if v.shape[0] > 0 else 0)
+    if (v.shape[0] > 0 and v[0].numel() != C) or v.shape[0] < int(n) or idx.numel() < int(n):
+        raise ValueError("v must hold n rows of z's row size; idx n entries")
+    if zc is None:
+        zc = torch.empty((max(int(n), 1),) + tuple(z.shape[1:]), dtype=z.dtype, device=z.device)
+    if not zc.is_contiguous() or zc.dtype != z.dtype or zc.shape[0] < int(n) or (zc.shape[0] and zc[0].numel() != C):
+        raise ValueError("zc must be contiguous with n rows of z's row size and dtype")
+    dtype = UT_BF16 if z.dtype == torch.bfloat16 else UT_F32
+    st = lib().ut_fg_euler_update_gather(_p(idx), int(n), _p(z), _p(v), _p(zc), T, C, dtype, float(dt), _p(status),
+                                         _stream())
+    _check("ut_fg_euler_update_gather", st)
+    return zc
 
 
 def ut_fg_composite(mask: torch.Tensor, z: torch.Tensor, z_bg: torch.Tensor) -> None:

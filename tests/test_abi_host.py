@@ -141,6 +141,13 @@ def test_sampler_argument_errors_are_caught_on_host(L):
     assert f(None, 5, bogus, bogus, 10, 64, u.UT_F32, 0.5, None, None) == u.UT_ERR_INVALID_ARG
     # n = 0 is a no-op (nothing is dereferenced)
     assert f(None, 0, None, None, 10, 64, u.UT_BF16, 0.5, None, None) == u.UT_OK
+    fg = L.ut_fg_euler_update_gather
+    # the fused gather: same checks, plus a missing or misaligned zc
+    assert fg(bogus, 11, bogus, bogus, bogus, 10, 64, u.UT_BF16, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert fg(bogus, 5, bogus, bogus, None, 10, 64, u.UT_BF16, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert fg(bogus, 5, bogus, bogus, odd, 10, 64, u.UT_BF16, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert fg(bogus, 5, bogus, bogus, bogus, 10, 12, u.UT_BF16, 0.5, None, None) == u.UT_ERR_INVALID_ARG
+    assert fg(None, 0, None, None, None, 10, 64, u.UT_BF16, 0.5, None, None) == u.UT_OK
     g = L.ut_fg_composite
     assert g(bogus, 10, bogus, bogus, 0, 128, None) == u.UT_ERR_INVALID_ARG      # empty tile
     assert g(bogus, 10, bogus, bogus, 4, 100, None) == u.UT_ERR_INVALID_ARG      # row not 16-byte multiple

@@ -138,3 +138,29 @@ def test_composite_all_foreground_and_all_background():
         u.ut_fg_composite(torch.from_numpy(m).cuda(), z, tile.cuda())
         torch.cuda.synchronize()
         assert np.array_equal(bits(z.cpu()), o.fg_composite(bits(z0), m, bits(tile)))
+
+
+@pytest.mark.parametrize("cfg", ["c512", "c2048"])
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_euler_update_gather_matches_oracle(cfg, dtype):
+    """The Euler step fused with the next step's gather: the canvas rows as in
+    ut_fg_euler_update (within the rounding bound of the oracle, background
+    untouched) and zc[n] = the updated z[idx[n]] bit for bit."""
+    need_gpu()
+    from paper_2609_23169_gb300 import ultratex as u
+    x = _inputs(cfg, dtype)
+    idx = np.nonzero(x["mask"])[0].astype(np.int32)
+    n = len(idx)
+    dt = float(np.float32(x["dt"]))
+    z0, v = x["z"], x["v"]
+    z = z0.cuda()
+    z_ref = z0.cuda()
+    ti = torch.from_numpy(idx).cuda()
+    st = u.status_word()
+    zc = u.ut_fg_euler_update_gather(ti, n, z, v.cuda(), dt, status=st)
+    u.ut_fg_euler_update(ti, n, z_ref, v.cuda(), dt, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    _check_euler(z0, z, idx, v, dt, dtype)
+    assert np.array_equal(bits(z), bits(z_ref))            # same canvas as the unfused step
+    assert np.array_equal(bits(zc[:n]), bits(z[ti]))       # the gather of the updated rows
