@@ -167,39 +167,6 @@ UT_DEV void red_add_f32(float* p, float v) {
   asm volatile("red.relaxed.gpu.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
 }
 
-// The query steps of an item.  kMode 0: 128-row blocks on both sides; 1:
-// 128-row query blocks, 64-row key blocks (merged lists, TileList); 2: 64-row
-// query blocks paired into 128-row tiles (PairList, one list); 3: 64-row
-// blocks on both sides, per item whichever of the merged tiles and the paired
-// lists takes fewer steps.  next() gives the tile's query blocks (paired: the
-// 64-row blocks of the low and high halves, -1 if missing; merged: lo = the
-// 128-row query tile) and the visibility bits.  In mode 3 init() takes the
-// item's choice from the lists' first and last entries (pairing_is_shorter),
-// the same in every role.
-template <int kMode>
-struct QuerySteps {
-  TileList<kMode == 1 || kMode == 3> tl;
-  PairList pl;
-  bool pair;
-  UT_DEV void init(const BwdParams& prm, int h, int j) {
-    if (kMode != 2) tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
-    if (kMode == 2) pl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile == 2);
-    pair = kMode == 2;
-    if constexpr (kMode == 3) pair = pairing_is_shorter(tl);
-  }
-  UT_DEV int count_warp() const {
-    if (kMode == 3 && pair) return tl.na > tl.nb ? tl.na : tl.nb;
-    return kMode == 2 ? pl.count() : tl.count_warp();
-  }
-  UT_DEV bool empty() const { return kMode == 2 ? pl.empty() : tl.empty(); }
-  UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
-    if (kMode == 2) return pl.next(lo, hi, bits);
-    if (kMode == 3 && pair) return PairList::step_two(tl.a, tl.b, tl.na, tl.nb, tl.pa, lo, hi, bits);
-    hi = -1;
-    return tl.next(lo, bits);
-  }
-};
-
 template <int D, int kMode>
 __global__ void __launch_bounds__(kFuThreads, 1)
     bwd_fused_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -320,8 +287,8 @@ __global__ void __launch_bounds__(kFuThreads, 1)
           }
           if (w < 0) break;
           const int h = w / prm.nq, j = w % prm.nq;
-          QuerySteps<kMode> tl;
-          tl.init(prm, h, j);
+          BlockSteps<kMode> tl;
+          tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
           if (tl.empty()) continue;
           if (is_q) {
             if (!(ok = mbar_wait(&sm.kv_empty, (ki & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -372,8 +339,8 @@ __global__ void __launch_bounds__(kFuThreads, 1)
         for (;;) {
           int w;
           if (!(ok = next_item(kk, w, false)) || w < 0) break;
-          QuerySteps<kMode> tl;
-          tl.init(prm, w / prm.nq, w % prm.nq);
+          BlockSteps<kMode> tl;
+          tl.init(prm.ptr, prm.idx, w / prm.nq, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
           const int L = tl.count_warp();
           if (L <= 0) continue;
           if (!(ok = warp_wait(&sm.kv_full, ki & 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -474,8 +441,8 @@ __global__ void __launch_bounds__(kFuThreads, 1)
       int w;
       if (!(ok = next_item(kk, w, false)) || w < 0) break;
       const int h = w / prm.nq, j = w % prm.nq;
-      QuerySteps<kMode> tl;
-      tl.init(prm, h, j);
+      BlockSteps<kMode> tl;
+      tl.init(prm.ptr, prm.idx, h, j, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
       const int L = tl.count_warp();
       const int64_t gk = (int64_t)j * kTile + krow;
       const bool row_ok = gk < prm.N;
@@ -634,8 +601,8 @@ __global__ void __launch_bounds__(kFuThreads, 1)
       int w;
       if (!(ok = next_item(kk, w, false)) || w < 0) break;
       const int h = w / prm.nq;
-      QuerySteps<kMode> tl;
-      tl.init(prm, h, w % prm.nq);
+      BlockSteps<kMode> tl;
+      tl.init(prm.ptr, prm.idx, h, w % prm.nq, prm.nk_fine, prm.k_rows_per_tile, prm.list_shift);
       const int L = tl.count_warp();
       if (L <= 0) continue;
       for (int t = 0; t < L; ++t) {

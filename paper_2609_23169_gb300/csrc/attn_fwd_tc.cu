@@ -86,41 +86,6 @@ struct FwdParams {
   uint64_t timeout_ns;
 };
 
-// The key steps of an item.  kMode 0: 128-row blocks on both sides (the list
-// itself); 1: 64-row query blocks, 128-row key blocks (the item's two lists
-// merged, TileList); 2: 64-row key blocks paired into 128-row tiles
-// (PairList); 3: 64-row blocks on both sides, per item whichever of the
-// merged tiles and the paired lists takes fewer steps (pairing discards half
-// of each tile but merging discards the unlisted sub-blocks, most of them
-// when the lists are sparse; dense or clustered lists merge into fewer
-// tiles).  next() gives the tile's key blocks (paired: the 64-row blocks of
-// the low and high halves, -1 if missing; merged: lo = the 128-row key tile)
-// and the visibility bits.  In mode 3 init() takes the item's choice from the
-// lists' first and last entries (pairing_is_shorter), the same in every role.
-template <int kMode>
-struct KeySteps {
-  TileList<kMode == 1 || kMode == 3> tl;
-  PairList pl;
-  bool pair;
-  UT_DEV void init(const FwdParams& prm, int h, int i) {
-    if (kMode != 2) tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
-    if (kMode == 2) pl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile == 2);
-    pair = kMode == 2;
-    if constexpr (kMode == 3) pair = pairing_is_shorter(tl);
-  }
-  UT_DEV int count_warp() const {
-    if (kMode == 3 && pair) return tl.na > tl.nb ? tl.na : tl.nb;
-    return kMode == 2 ? pl.count() : tl.count_warp();
-  }
-  UT_DEV bool empty() const { return kMode == 2 ? pl.empty() : tl.empty(); }
-  UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
-    if (kMode == 2) return pl.next(lo, hi, bits);
-    if (kMode == 3 && pair) return PairList::step_two(tl.a, tl.b, tl.na, tl.nb, tl.pa, lo, hi, bits);
-    hi = -1;
-    return tl.next(lo, bits);
-  }
-};
-
 template <int D, int kMode>
 __global__ void __launch_bounds__(kFwdThreads, 1)
     attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -192,8 +157,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
         const int h = w / prm.nq, i = w % prm.nq;
-        KeySteps<kMode> tl;
-        tl.init(prm, h, i);
+        BlockSteps<kMode> tl;
+        tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
         if (tl.empty()) continue;
         if (is_k) {
           if (!(ok = mbar_wait(&sm.q_empty, (qi & 1) ^ 1, abort_flag, prm.status, prm.timeout_ns))) break;
@@ -239,8 +204,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       uint32_t qi = 0, oi = 0, kv0 = 0, sc0 = 0;
       bool ok = true;
       for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
-        KeySteps<kMode> tl;
-        tl.init(prm, w / prm.nq, w % prm.nq);
+        BlockSteps<kMode> tl;
+        tl.init(prm.row_ptr, prm.col_idx, w / prm.nq, w % prm.nq, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
         const int L = tl.count_warp();
         if (L <= 0) continue;
         // Q of this item in TMEM (the softmax warps copied it there)
@@ -374,8 +339,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     };
     for (int w = blockIdx.x; w < prm.n_items && ok; w += G) {
       const int h = w / prm.nq, i = w % prm.nq;
-      KeySteps<kMode> tl;
-      tl.init(prm, h, i);
+      BlockSteps<kMode> tl;
+      tl.init(prm.row_ptr, prm.col_idx, h, i, prm.nq_fine, prm.q_rows_per_tile, prm.list_shift);
       const int L = tl.count_warp();
       const int64_t grow = (int64_t)i * kBM + row;
       if (L <= 0) {

@@ -388,6 +388,44 @@ UT_DEV bool pairing_is_shorter(const TileList<true>& tl) {
   return paired < (spanned < entries ? spanned : entries);
 }
 
+// The steps of an item over the listed side.  kMode 0: 128-row blocks on both
+// sides (the list itself); 1: 64-row blocks on the item's side, 128-row
+// blocks listed (the item's two lists merged, TileList); 2: 64-row blocks
+// listed, 128-row item blocks (consecutive entries paired, PairList); 3:
+// 64-row blocks on both sides, per item whichever of the merged tiles and the
+// two lists in lockstep takes fewer steps (pairing_is_shorter, decided in
+// init() from the lists' first and last entries, the same in every role).
+// next() gives the tile's listed blocks (paired: the 64-row blocks of the low
+// and high halves, -1 if missing; merged or plain: lo = the 128-row tile) and
+// the visibility bits.
+template <int kMode>
+struct BlockSteps {
+  TileList<kMode == 1 || kMode == 3> tl;
+  PairList pl;
+  bool pair;
+  // item = 128-row block t of head h on the item's side; ptr/idx the fine
+  // lists with nfine rows per head; rows_per_tile = 2 for 64-row blocks on the
+  // item's side; list_shift = 1 for 64-row listed blocks
+  UT_DEV void init(const int32_t* ptr, const int32_t* idx, int h, int t, int nfine, int rows_per_tile,
+                   int list_shift) {
+    if (kMode != 2) tl.init(ptr, idx, h, t, nfine, rows_per_tile, list_shift);
+    if (kMode == 2) pl.init(ptr, idx, h, t, nfine, rows_per_tile == 2);
+    pair = kMode == 2;
+    if constexpr (kMode == 3) pair = pairing_is_shorter(tl);
+  }
+  UT_DEV int count_warp() const {
+    if (kMode == 3 && pair) return tl.na > tl.nb ? tl.na : tl.nb;
+    return kMode == 2 ? pl.count() : tl.count_warp();
+  }
+  UT_DEV bool empty() const { return kMode == 2 ? pl.empty() : tl.empty(); }
+  UT_DEV bool next(int& lo, int& hi, uint32_t& bits) {
+    if (kMode == 2) return pl.next(lo, hi, bits);
+    if (kMode == 3 && pair) return PairList::step_two(tl.a, tl.b, tl.na, tl.nb, tl.pa, lo, hi, bits);
+    hi = -1;
+    return tl.next(lo, bits);
+  }
+};
+
 // ---------------------------------------------------------------- tcgen05
 UT_DEV void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
