@@ -930,8 +930,12 @@ def main():
     if rank == 0:
         if not args.no_cpu_baseline and world == 1:
             v, desc, dt = oracle_sample(w, args.cpu_seconds)
+            step_tflop = 3.5 * line["retained_fwd_tflop"]
             line["cpu_baseline"] = {"value": round(v, 6), "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
-                                    "sample": desc + f" ({dt:.1f} s)"}
+                                    "sample": desc + f" ({dt:.1f} s)",
+                                    "extrapolated_step_s": round(step_tflop / v, 1),
+                                    "extrapolation": "the whole step's retained-pair work (forward + backward, "
+                                                     f"{step_tflop:.2f} TFLOP) at the sample's rate; not measured"}
         if not args.no_oracle_times and world == 1:
             line["oracle_times"] = oracle_wall_times(cpu_cores())
         print(json.dumps(line))

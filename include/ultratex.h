@@ -64,9 +64,11 @@ enum { UT_MASK_TOPK = 0, UT_MASK_BITMAP = 1 };
  * key blocks of b_kv = block_k rows (block_k = 0: b_kv = b_q).
  * N_q = ceil(N / b_q), N_k = ceil(N / b_kv); the last block may be partial
  * (its missing key rows are excluded, its missing query rows are not
- * written).  The bf16 tensor-core kernels work on 128 x 128 tiles; with 64-row
- * blocks a tile holds two of them and the pairs not listed inside a listed
- * tile are masked out (their work is computed and discarded). */
+ * written).  The bf16 tensor-core kernels work on 128 x 128 tiles; a 64-row
+ * block fills half of a tile: two listed 64-row blocks share one operand
+ * tile, or, for 64-row blocks on both sides, an item's lists are merged into
+ * 128-row tiles when that takes fewer tiles; work on the parts of a tile that
+ * no listed pair covers is computed and discarded. */
 typedef struct {
   int64_t n_tokens;    /* N: rows of the compacted sequence, >= 0 */
   int32_t n_heads;     /* H >= 1 */

@@ -61,8 +61,12 @@ def _gpu_fwd_bwd(q, k, v, do, lists, bq, bk):
 
 
 @pytest.mark.parametrize("bq,bk", COMBOS)
-@pytest.mark.parametrize("N,H,d,dens,seed", [(300, 2, 128, 0.5, 1), (1000, 2, 128, 0.25, 2), (700, 1, 64, 0.4, 3)])
+@pytest.mark.parametrize("N,H,d,dens,seed", [(300, 2, 128, 0.5, 1), (1000, 2, 128, 0.25, 2), (700, 1, 64, 0.4, 3),
+                                             (1500, 2, 128, 0.9, 4), (2100, 2, 128, 0.06, 5)])
 def test_bitmap_lists_full(bq, bk, N, H, d, dens, seed):
+    # dense (0.9) and sparse (0.06) lists take both forms of the 64-row
+    # handling (merged tiles, paired blocks); lists of unequal lengths leave
+    # one half of some paired tiles empty.
     # one 64-row query block with an empty list: its rows see nothing (O = 0, LSE = -inf)
     empty = [(0, 1)] if bq == 64 else [(0, 0)]
     q, k, v, do, bm = _bitmap_problem(N, H, d, bq, bk, dens, seed, empty)
